@@ -1,0 +1,185 @@
+/*
+ * psppo.h -- C ABI of the GB300 (sm_103a) PS-PPO LM-head update pass.
+ *
+ * The update pass of Prefix-Sampling PPO (Algorithm 1, steps 6 and 10-11) over the
+ * LM head: per-completion cutoffs H ~ xi with inverse-survival weights 1/xi_t
+ * (Section 3.2), ragged packing of the retained prefixes with group-normalised
+ * advantages (Section 3.1), the weighted clipped PPO surrogate through the head
+ * (Eq. 1, Eq. truncated_update_Ghat) and its gradients dH and dW (Appendix D).
+ *
+ * Conventions shared by every entry point:
+ *  - All array pointers are DEVICE pointers owned by the caller, except where an
+ *    argument is documented as a host pointer. The library allocates no device
+ *    memory; scratch is the caller's workspace `ws` of `ws_bytes` bytes (at least
+ *    the matching *_workspace_size(); 256-byte aligned).
+ *  - Every call is asynchronous and ordered on `stream` (a cudaStream_t; NULL is
+ *    the legacy default stream), unless a host output is requested.
+ *  - Every call returns a ps_status (0 = PS_OK). Arguments are checked on the host
+ *    before anything is launched; a failed check launches nothing.
+ *  - Data that can only be checked on the device (masses that do not sum to 2^62,
+ *    a length out of range, a token id outside [0, V), more rows than capacity, a
+ *    barrier wait that ran out of time) set bits in a status word at the start of
+ *    the call's workspace. Each call clears that word when it starts;
+ *    ps_workspace_status() synchronises the stream and reports it.
+ *  - Row-major layouts. "bf16" is IEEE bfloat16, "f32" IEEE binary32.
+ *  - No global state: calls on different streams with different workspaces may
+ *    run concurrently.
+ */
+#ifndef PSPPO_H_
+#define PSPPO_H_
+
+#include <stddef.h>
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+typedef struct CUstream_st* ps_stream_t; /* identical to cudaStream_t */
+
+typedef enum {
+  PS_OK = 0,
+  PS_ERR_INVALID_ARG = 1,   /* a host-checked argument is out of range or NULL */
+  PS_ERR_UNSUPPORTED = 2,   /* dtype, shape or device not supported (e.g. not sm_103) */
+  PS_ERR_WORKSPACE = 3,     /* ws_bytes smaller than the required size, or ws misaligned */
+  PS_ERR_CAPACITY = 4,      /* (device) more packed rows than the given capacity */
+  PS_ERR_DEVICE_DATA = 5,   /* (device) bad masses, lengths or token ids */
+  PS_ERR_TIMEOUT = 6,       /* (device) a bounded wait inside a kernel ran out */
+  PS_ERR_CUDA = 7           /* a CUDA runtime call failed */
+} ps_status;
+
+enum { PS_MODE_TRUNC = 0, PS_MODE_FULL = 1 };
+enum { PS_DTYPE_BF16 = 0, PS_DTYPE_F32 = 1 };
+enum { PS_ADV_CENTERED = 0, PS_ADV_GROUP_NORM = 1 };
+enum { PS_DW_OVERWRITE = 0, PS_DW_ACCUMULATE = 1 };
+
+/* Device status bits (the word at offset 0 of every workspace). */
+enum {
+  PS_DEV_BAD_PMF = 1, PS_DEV_BAD_LENGTH = 2, PS_DEV_CAPACITY = 4,
+  PS_DEV_BAD_TOKEN = 8, PS_DEV_TIMEOUT = 16
+};
+
+/* Static string for a ps_status value. */
+const char* ps_status_string(int status);
+
+/* Library ABI version (major * 10000 + minor * 100 + patch). */
+int ps_version(void);
+
+/*
+ * Synchronise `stream`, read the device status word of a workspace used by a
+ * previous call on that stream, and map it to a ps_status (PS_OK if clear). If
+ * `bits` is not NULL (host pointer) the raw PS_DEV_* bits are stored there.
+ */
+int ps_workspace_status(const void* ws, ps_stream_t stream, uint32_t* bits);
+
+/* ---------------------------------------------------------------------------
+ * ps_sample_cutoffs -- cutoffs and inverse-survival weights.
+ *
+ * Section 3.2: the cutoff H of a completion has survival xi_t = Pr(H >= t | x);
+ * tokens t <= H are kept and reweighted by 1/xi_t (Eq. truncated_update_Ghat,
+ * Algorithm 1 steps 10-11, unbiased by Appendix B).
+ *
+ * q      [P][T_max] uint64 masses: Pr(H = h) = q[p][h-1] / 2^62 for prompt p; each
+ *        row must sum to exactly 2^62 (checked on the device: PS_DEV_BAD_PMF).
+ * L      [B] int32 completion lengths, 1 <= L <= T_max (PS_DEV_BAD_LENGTH), B = P*K;
+ *        completion k belongs to prompt k / K.
+ * seed, step, traj_base: the cutoff of completion k is decided by the 62-bit
+ *        uniform x = (Philox4x64-10(counter = (traj_base + k, step, 0, 0),
+ *        key = (seed, 0x5053505030303031))[0]) >> 2, as H = min{h : x < U[h]},
+ *        U[h] = q[p][0] + ... + q[p][h-1]. traj_base is the global index of the
+ *        first completion, so a batch split across ranks draws the same cutoffs.
+ * mode   PS_MODE_TRUNC, or PS_MODE_FULL (H = L, weights 1: the untruncated control).
+ * H, n   [B] int32 outputs: the cutoff and the prefix length n = min(H, L).
+ * w_tab  [P][T_max] f32 output: w_tab[p][t-1] = 2^62 / S_p[t] rounded to f32, with
+ *        S_p[t] = 2^62 - U_p[t-1] (so 1/w = xi_t exactly before rounding); +inf
+ *        where S_p[t] = 0 (never read); 1 in full mode.
+ * Limits: 1 <= K <= 8192, 1 <= T_max <= 2^24, P >= 1.
+ * ------------------------------------------------------------------------- */
+size_t ps_sample_cutoffs_workspace_size(int P, int K, int T_max);
+int ps_sample_cutoffs(int P, int K, int T_max, const uint64_t* q, const int32_t* L,
+                      uint64_t seed, uint64_t step, int64_t traj_base, int mode,
+                      int32_t* H, int32_t* n, float* w_tab,
+                      void* ws, size_t ws_bytes, ps_stream_t stream);
+
+/* ---------------------------------------------------------------------------
+ * ps_pack_prefixes -- group advantages and the packed prefix rows.
+ *
+ * Section 3.1: one advantage per completion, A = R - mean_group(R)
+ * (PS_ADV_CENTERED) or (R - mean) / (std + 1e-6) with the population std
+ * (PS_ADV_GROUP_NORM); group sums run sequentially in f64. Algorithm 1 step 11:
+ * only tokens t <= n_k are kept; rows (k, t), k = 0..B-1, t = 1..n_k are laid out
+ * back to back in that order.
+ *
+ * Inputs: L, n [B] int32 (as from ps_sample_cutoffs; 0 <= n <= L), R [B] f32
+ * rewards, w_tab [P][T_max] f32, tok_full [sum L] int32, oldlogp_full [sum L] f32,
+ * hid_full [sum L][d] (dtype; may be NULL to skip the hidden-state gather).
+ * capacity: rows available in every per-row output. If sum n > capacity the call
+ * writes no rows and sets PS_DEV_CAPACITY.
+ * Outputs: cu_seqlens [B+1] int32 (exclusive scan of n; cu_seqlens[B] = N);
+ * per row i < N: tok, oldlogp, w (= w_tab[k/K][t-1]), adv (= A_k, f32),
+ * hid_packed [N][d]; optional (may be NULL): src_row (row of the unpacked batch),
+ * row_traj (k), row_pos (t, 1-based).
+ * h_num_rows: HOST pointer; if not NULL the call synchronises the stream and
+ * stores N there.
+ * Limits: d % 8 == 0 (bf16) or d % 4 == 0 (f32); sum L < 2^31.
+ * ------------------------------------------------------------------------- */
+size_t ps_pack_prefixes_workspace_size(int P, int K);
+int ps_pack_prefixes(int P, int K, int T_max, int d, int dtype,
+                     const int32_t* L, const int32_t* n, const float* R, int adv_mode,
+                     const float* w_tab, const int32_t* tok_full, const float* oldlogp_full,
+                     const void* hid_full, int64_t capacity,
+                     int32_t* cu_seqlens, int32_t* src_row, int32_t* row_traj, int32_t* row_pos,
+                     int32_t* tok, float* oldlogp, float* w, float* adv, void* hid_packed,
+                     int64_t* h_num_rows, void* ws, size_t ws_bytes, ps_stream_t stream);
+
+/* ---------------------------------------------------------------------------
+ * ps_lmhead_ppo_fwd -- fused LM-head forward: loss without materialised logits.
+ *
+ * For each packed row i (Appendix D head, Eq. 1 surrogate):
+ *   z_i = W h_i (W stored [V][d]; f32 accumulation), lse_i = log sum_v exp(z_iv),
+ *   logp_i = z_{i,tok_i} - lse_i, ratio_i = exp(logp_i - oldlogp_i),
+ *   s_i = min(ratio_i adv_i, clip(ratio_i, 1-eps, 1+eps) adv_i),
+ *   row_loss_i = -loss_scale * w_i * s_i,   loss = sum_i row_loss_i (f64, fixed order),
+ *   coef_i = d loss / d logp_i = -loss_scale * w_i * adv_i * ratio_i, or 0 where the
+ *   clip binds ((adv > 0 and ratio > 1+eps) or (adv < 0 and ratio < 1-eps)).
+ * loss_scale is 1/(P*K) for the paper's estimator (1/K per prompt, mean over prompts).
+ *
+ * Hpk [N][d], W [V][d]: dtype PS_DTYPE_BF16 (tcgen05 tensor cores) or PS_DTYPE_F32
+ * (f32 CUDA cores). tok [N] int32 (0 <= tok < V, else PS_DEV_BAD_TOKEN), oldlogp,
+ * adv, w [N] f32. Outputs: loss [1] f64 (device), lse, logp, ratio, coef [N] f32,
+ * row_loss [N] f32 (may be NULL). Only O(N) values are written; the N x V logits
+ * are never stored.
+ * Limits: N >= 0 (N = 0 writes loss = 0), 1 <= V < 2^31, d % 8 == 0 (bf16) or
+ * d % 4 == 0 (f32); 16-byte aligned Hpk and W.
+ * ------------------------------------------------------------------------- */
+size_t ps_lmhead_ppo_fwd_workspace_size(int64_t N, int d, int V, int dtype);
+int ps_lmhead_ppo_fwd(int64_t N, int d, int V, int dtype, const void* Hpk, const void* W,
+                      const int32_t* tok, const float* oldlogp, const float* adv, const float* w,
+                      double eps, double loss_scale,
+                      double* loss, float* lse, float* logp, float* ratio, float* coef,
+                      float* row_loss, void* ws, size_t ws_bytes, ps_stream_t stream);
+
+/* ---------------------------------------------------------------------------
+ * ps_lmhead_ppo_bwd -- fused LM-head backward over recomputed logit tiles.
+ *
+ * Appendix D: d logp / dz = e_o - p. With coef from the forward:
+ *   dZ_iv = coef_i (1[v = tok_i] - exp(z_iv - lse_i)),
+ *   dH = dZ W            [N][d] f32 (overwritten),
+ *   dW = dZ^T Hpk        [V][d] f32 (overwritten, or added to with PS_DW_ACCUMULATE).
+ * The logits are recomputed tile by tile; dZ is held, in the operand dtype, only
+ * for one chunk of rows at a time inside the workspace: the chunk is the largest
+ * multiple of 128 rows that fits (ws_bytes), so a larger workspace means fewer
+ * chunks. dH or dW may be NULL to skip that product.
+ * Limits as for the forward; ws_bytes >= ps_lmhead_ppo_bwd_workspace_size(N, d, V,
+ * dtype, 128) (one chunk of 128 rows).
+ * ------------------------------------------------------------------------- */
+size_t ps_lmhead_ppo_bwd_workspace_size(int64_t N, int d, int V, int dtype, int64_t chunk_rows);
+int ps_lmhead_ppo_bwd(int64_t N, int d, int V, int dtype, const void* Hpk, const void* W,
+                      const int32_t* tok, const float* lse, const float* coef,
+                      float* dH, float* dW, int flags,
+                      void* ws, size_t ws_bytes, ps_stream_t stream);
+
+#ifdef __cplusplus
+}
+#endif
+#endif /* PSPPO_H_ */

@@ -1,0 +1,15 @@
+"""GB300-native (sm_103a) PS-PPO LM-head update pass.
+
+The computation lives in libpsppo.so (hand-written CUDA, tcgen05 tensor cores, TMA)
+behind the C ABI of include/psppo.h; this package is its ctypes binding (same names)
+plus UpdatePass, which holds the device buffers of one batch shape in torch.
+"""
+from ._binding import *  # noqa: F401,F403
+from ._binding import PsppoError, lib, status_string  # noqa: F401
+
+
+def __getattr__(name):
+    if name in ("UpdatePass", "PassShape"):
+        from . import pipeline
+        return getattr(pipeline, name)
+    raise AttributeError(name)

@@ -1,0 +1,38 @@
+// Internal interfaces between the translation units of libpsppo (not exported).
+#pragma once
+
+#include <cuda_runtime.h>
+#include <stdint.h>
+
+namespace psk {
+
+int num_sms_current();
+int device_is_sm103();
+
+// Forward GEMM with the online-logsumexp epilogue. part: [splits][N] (max2, sum) pairs
+// (max in log2 units); ztok: [N] chosen-token logit.
+int max_fwd_splits_bf16();
+int choose_fwd_splits_bf16(int64_t N, int V, int num_sms);
+int fwd_gemm_bf16(int64_t N, int d, int V, const void* Hpk, const void* W, const int32_t* tok, float2* part,
+                  float* ztok, int splits, uint32_t* status, cudaStream_t s);
+int fwd_splits_f32(int V);
+int fwd_gemm_f32(int64_t N, int d, int V, const float* Hpk, const float* W, const int32_t* tok, float2* part,
+                 float* ztok, uint32_t* status, cudaStream_t s);
+
+// Backward for one chunk of rows [0, rc) of already offset pointers: recompute dZ into
+// dz ([rc][ldz], operand dtype), then dH = dZ W and dW (+)= dZ^T Hpk.
+int bwd_chunk_bf16(int64_t rc, int d, int V, const void* Hpk, const void* W, const int32_t* tok,
+                   const float* lse, const float* coef, float* dH, float* dW, int dw_accumulate, void* dz,
+                   int64_t ldz, uint32_t* status, cudaStream_t s);
+int bwd_chunk_f32(int64_t rc, int d, int V, const float* Hpk, const float* W, const int32_t* tok,
+                  const float* lse, const float* coef, float* dH, float* dW, int dw_accumulate, float* dz,
+                  int64_t ldz, uint32_t* status, cudaStream_t s);
+
+// Plain tensor-core GEMM (test hook): C[M][N] (+)= sum_k A(m,k) B(k,n), f32 out.
+int gemm_bf16(int M, int N, int K, int a_mn, int b_mn, const void* A, int64_t lda, const void* B, int64_t ldb,
+              float* C, int64_t ldc, int accumulate, uint32_t* status, cudaStream_t s);
+
+// Bounded-wait self test: waits on an mbarrier nobody arrives at.
+int wait_timeout_probe(uint64_t timeout_ns, uint32_t* status, cudaStream_t s);
+
+}  // namespace psk

@@ -1,0 +1,320 @@
+// bf16 LM-head forward/backward on the tcgen05 tensor cores (sm_103a).
+//
+// Forward (Eq. 1 through the head of Appendix D): Z = Hpk W^T tile by tile; the
+// epilogue folds each 32-column slice into a per-row running (max, sum of exp) in
+// log2 units and captures the chosen token's logit, so the N x V logits never leave
+// TMEM. Backward: the same product is recomputed per chunk of rows and turned into
+// dZ = coef (onehot - softmax) in bf16; dH = dZ W and dW = dZ^T Hpk are two more
+// tensor-core products over that chunk.
+#include <mutex>
+
+#include <cuda_bf16.h>
+
+#include "internal.h"
+#include "umma_gemm.cuh"
+
+namespace psk {
+
+// ============================================================================= epilogues
+struct FwdLseEpi {
+  struct Params {
+    const int32_t* tok;
+    int M, N;
+    float2* part;
+    float* ztok;
+  };
+  struct State {
+    float m2, s;
+    int tok;
+  };
+  static __device__ __forceinline__ void begin_unit(const Params& p, State& st, int row, int) {
+    st.m2 = -INFINITY;
+    st.s = 0.f;
+    st.tok = row < p.M ? __ldg(p.tok + row) : -1;
+  }
+  static __device__ __forceinline__ void chunk(const Params& p, State& st, int row, int col0,
+                                               const uint32_t (&r)[32]) {
+    if (col0 >= p.N) return;
+    float x[32];
+    const int nv = p.N - col0;
+#pragma unroll
+    for (int j = 0; j < 32; ++j) x[j] = (j < nv) ? __uint_as_float(r[j]) * kLog2e : -INFINITY;
+    float c0 = fmaxf(x[0], x[1]), c1 = fmaxf(x[2], x[3]);
+#pragma unroll
+    for (int j = 4; j < 32; j += 4) {
+      c0 = fmaxf(c0, fmaxf(x[j], x[j + 1]));
+      c1 = fmaxf(c1, fmaxf(x[j + 2], x[j + 3]));
+    }
+    const int rel = st.tok - col0;
+    if (static_cast<unsigned>(rel) < 32u) {
+      float zt = 0.f;
+#pragma unroll
+      for (int j = 0; j < 32; ++j)
+        if (j == rel) zt = __uint_as_float(r[j]);
+      p.ztok[row] = zt;
+    }
+    const float mn = fmaxf(st.m2, fmaxf(c0, c1));
+    float a0 = 0.f, a1 = 0.f, a2 = 0.f, a3 = 0.f;
+#pragma unroll
+    for (int j = 0; j < 32; j += 4) {
+      a0 += exp2f(x[j] - mn);
+      a1 += exp2f(x[j + 1] - mn);
+      a2 += exp2f(x[j + 2] - mn);
+      a3 += exp2f(x[j + 3] - mn);
+    }
+    st.s = st.s * exp2f(st.m2 - mn) + ((a0 + a1) + (a2 + a3));
+    st.m2 = mn;
+  }
+  static __device__ __forceinline__ void end_unit(const Params& p, State& st, int row, int split) {
+    if (row < p.M) p.part[static_cast<size_t>(split) * p.M + row] = make_float2(st.m2, st.s);
+  }
+};
+
+struct BwdDzEpi {
+  struct Params {
+    const int32_t* tok;
+    const float* lse;
+    const float* coef;
+    int M, N;
+    __nv_bfloat16* dz;
+    int64_t ldz;
+  };
+  struct State {
+    float lse2, coef;
+    int tok;
+  };
+  static __device__ __forceinline__ void begin_unit(const Params& p, State& st, int row, int) {
+    if (row < p.M) {
+      st.tok = __ldg(p.tok + row);
+      st.lse2 = __ldg(p.lse + row) * kLog2e;
+      st.coef = __ldg(p.coef + row);
+    } else {
+      st.tok = -1;
+      st.lse2 = 0.f;
+      st.coef = 0.f;
+    }
+  }
+  static __device__ __forceinline__ void chunk(const Params& p, State& st, int row, int col0,
+                                               const uint32_t (&r)[32]) {
+    if (row >= p.M || col0 >= p.N) return;
+    uint32_t pk[16];
+    if (st.coef == 0.f) {
+#pragma unroll
+      for (int j = 0; j < 16; ++j) pk[j] = 0u;
+    } else {
+      const int rel = st.tok - col0;
+#pragma unroll
+      for (int j = 0; j < 16; ++j) {
+        const float p0 = exp2f(fmaf(__uint_as_float(r[2 * j]), kLog2e, -st.lse2));
+        const float p1 = exp2f(fmaf(__uint_as_float(r[2 * j + 1]), kLog2e, -st.lse2));
+        const float d0 = fmaf(-st.coef, p0, rel == 2 * j ? st.coef : 0.f);
+        const float d1 = fmaf(-st.coef, p1, rel == 2 * j + 1 ? st.coef : 0.f);
+        pk[j] = pack_bf16x2(d0, d1);
+      }
+    }
+    __nv_bfloat16* dst = p.dz + static_cast<int64_t>(row) * p.ldz + col0;
+    if (col0 + 32 <= p.N) {
+      uint4* d4 = reinterpret_cast<uint4*>(dst);
+#pragma unroll
+      for (int q = 0; q < 4; ++q) d4[q] = make_uint4(pk[4 * q], pk[4 * q + 1], pk[4 * q + 2], pk[4 * q + 3]);
+    } else {
+      const int nv = p.N - col0;
+      unsigned short* d16 = reinterpret_cast<unsigned short*>(dst);
+#pragma unroll
+      for (int j = 0; j < 32; ++j)
+        if (j < nv) d16[j] = static_cast<unsigned short>((j & 1) ? (pk[j >> 1] >> 16) : (pk[j >> 1] & 0xFFFFu));
+    }
+  }
+  static __device__ __forceinline__ void end_unit(const Params&, State&, int, int) {}
+};
+
+struct StoreF32Epi {
+  struct Params {
+    float* out;
+    int64_t ld;
+    int M, N;
+    int accumulate;
+  };
+  struct State {};
+  static __device__ __forceinline__ void begin_unit(const Params&, State&, int, int) {}
+  static __device__ __forceinline__ void chunk(const Params& p, State&, int row, int col0, const uint32_t (&r)[32]) {
+    if (row >= p.M || col0 >= p.N) return;
+    float* dst = p.out + static_cast<int64_t>(row) * p.ld + col0;
+    if (col0 + 32 <= p.N) {
+      float4* d4 = reinterpret_cast<float4*>(dst);
+#pragma unroll
+      for (int q = 0; q < 8; ++q) {
+        float4 v = make_float4(__uint_as_float(r[4 * q]), __uint_as_float(r[4 * q + 1]),
+                               __uint_as_float(r[4 * q + 2]), __uint_as_float(r[4 * q + 3]));
+        if (p.accumulate) {
+          const float4 o = d4[q];
+          v.x += o.x;
+          v.y += o.y;
+          v.z += o.z;
+          v.w += o.w;
+        }
+        d4[q] = v;
+      }
+    } else {
+      const int nv = p.N - col0;
+#pragma unroll
+      for (int j = 0; j < 32; ++j)
+        if (j < nv) dst[j] = (p.accumulate ? dst[j] : 0.f) + __uint_as_float(r[j]);
+    }
+  }
+  static __device__ __forceinline__ void end_unit(const Params&, State&, int, int) {}
+};
+
+// ============================================================================= host side
+typedef CUresult (*EncodeTiledFn)(CUtensorMap*, CUtensorMapDataType, cuuint32_t, void*, const cuuint64_t*,
+                                  const cuuint64_t*, const cuuint32_t*, const cuuint32_t*, CUtensorMapInterleave,
+                                  CUtensorMapSwizzle, CUtensorMapL2promotion, CUtensorMapFloatOOBfill);
+
+static EncodeTiledFn encode_fn() {
+  static EncodeTiledFn fn = nullptr;
+  static std::once_flag once;
+  std::call_once(once, [] {
+    void* p = nullptr;
+    cudaDriverEntryPointQueryResult q;
+    if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &p, 12000, cudaEnableDefault, &q) ==
+            cudaSuccess &&
+        q == cudaDriverEntryPointSuccess)
+      fn = reinterpret_cast<EncodeTiledFn>(p);
+  });
+  return fn;
+}
+
+// 2-D bf16 tensor [outer][inner] with row pitch `pitch_bytes`, 128-byte swizzled boxes.
+static bool make_map(CUtensorMap* m, const void* base, uint64_t inner, uint64_t outer, uint64_t pitch_bytes,
+                     uint32_t box_inner, uint32_t box_outer) {
+  EncodeTiledFn enc = encode_fn();
+  if (!enc) return false;
+  if ((reinterpret_cast<uintptr_t>(base) & 15) || (pitch_bytes & 15)) return false;
+  const cuuint64_t dims[2] = {inner, outer};
+  const cuuint64_t strides[1] = {pitch_bytes};
+  const cuuint32_t box[2] = {box_inner, box_outer};
+  const cuuint32_t estr[2] = {1, 1};
+  return enc(m, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<void*>(base), dims, strides, box, estr,
+             CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+             CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
+}
+
+// Operand maps. K-major [rows][K]: box 64 (K) x rows_box. MN-major [K][MN]: box 64 x 64.
+static bool map_kmajor(CUtensorMap* m, const void* base, int64_t rows, int64_t K, int64_t pitch_elems,
+                       uint32_t rows_box) {
+  return make_map(m, base, K, rows, pitch_elems * 2, kBK, rows_box);
+}
+static bool map_mnmajor(CUtensorMap* m, const void* base, int64_t K, int64_t MN, int64_t pitch_elems) {
+  return make_map(m, base, MN, K, pitch_elems * 2, 64, kBK);
+}
+
+template <bool A_MN, bool B_MN, class Epi>
+static int launch_gemm(const CUtensorMap& ta, const CUtensorMap& tb, int64_t M, int64_t N, int64_t K, int splits,
+                       int band_m, const typename Epi::Params& ep, uint32_t* status, cudaStream_t s) {
+  Sched sc;
+  sc.m_blocks = static_cast<int>((M + kBM - 1) / kBM);
+  sc.n_blocks = static_cast<int>((N + kBN - 1) / kBN);
+  sc.splits = splits > 0 ? splits : sc.n_blocks;
+  sc.band_m = band_m > 0 ? band_m : 1;
+  sc.num_units = sc.m_blocks * sc.splits;
+  sc.num_kb = static_cast<int>((K + kBK - 1) / kBK);
+  if (sc.num_units == 0) return PS_OK;
+  if (sc.num_kb == 0) return PS_ERR_INVALID_ARG;
+  auto kern = umma_gemm_kernel<A_MN, B_MN, Epi>;
+  if (cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, static_cast<int>(kGemmSmemBytes)) !=
+      cudaSuccess)
+    return PS_ERR_CUDA;
+  const int grid = sc.num_units < num_sms_current() ? sc.num_units : num_sms_current();
+  kern<<<grid, kGemmThreads, kGemmSmemBytes, s>>>(ta, tb, sc, ep, status, kDefaultTimeoutNs);
+  return cudaGetLastError() == cudaSuccess ? PS_OK : PS_ERR_CUDA;
+}
+
+constexpr int kMaxFwdSplits = 16;
+int max_fwd_splits_bf16() { return kMaxFwdSplits; }
+
+// Pick the number of vocabulary ranges per 128-row block that minimises the number of
+// tile rounds of a static round-robin over `num_sms` CTAs (smaller on ties).
+int choose_fwd_splits_bf16(int64_t N, int V, int num_sms) {
+  const int64_t mb = (N + kBM - 1) / kBM;
+  const int64_t nb = (V + kBN - 1) / kBN;
+  int best = 1;
+  int64_t best_cost = INT64_MAX;
+  for (int s = 1; s <= kMaxFwdSplits && s <= nb; ++s) {
+    const int64_t units = mb * s;
+    const int64_t rounds = (units + num_sms - 1) / num_sms;
+    const int64_t cost = rounds * ((nb + s - 1) / s);
+    if (cost < best_cost) {
+      best_cost = cost;
+      best = s;
+    }
+  }
+  return best;
+}
+
+int fwd_gemm_bf16(int64_t N, int d, int V, const void* Hpk, const void* W, const int32_t* tok, float2* part,
+                  float* ztok, int splits, uint32_t* status, cudaStream_t s) {
+  CUtensorMap ta, tb;
+  if (!map_kmajor(&ta, Hpk, N, d, d, kBM) || !map_kmajor(&tb, W, V, d, d, kBN)) return PS_ERR_INVALID_ARG;
+  FwdLseEpi::Params ep{tok, static_cast<int>(N), V, part, ztok};
+  const int band = (num_sms_current() + splits - 1) / splits;
+  return launch_gemm<false, false, FwdLseEpi>(ta, tb, N, V, d, splits, band, ep, status, s);
+}
+
+int bwd_chunk_bf16(int64_t rc, int d, int V, const void* Hpk, const void* W, const int32_t* tok,
+                   const float* lse, const float* coef, float* dH, float* dW, int dw_accumulate, void* dz,
+                   int64_t ldz, uint32_t* status, cudaStream_t s) {
+  int rcode;
+  {
+    CUtensorMap ta, tb;
+    if (!map_kmajor(&ta, Hpk, rc, d, d, kBM) || !map_kmajor(&tb, W, V, d, d, kBN)) return PS_ERR_INVALID_ARG;
+    BwdDzEpi::Params ep{tok, lse, coef, static_cast<int>(rc), V, static_cast<__nv_bfloat16*>(dz), ldz};
+    rcode = launch_gemm<false, false, BwdDzEpi>(ta, tb, rc, V, d, 0, 16, ep, status, s);
+    if (rcode != PS_OK) return rcode;
+  }
+  if (dH) {
+    CUtensorMap ta, tb;
+    if (!map_kmajor(&ta, dz, rc, V, ldz, kBM) || !map_mnmajor(&tb, W, V, d, d)) return PS_ERR_INVALID_ARG;
+    StoreF32Epi::Params ep{dH, d, static_cast<int>(rc), d, 0};
+    rcode = launch_gemm<false, true, StoreF32Epi>(ta, tb, rc, d, V, 0, 16, ep, status, s);
+    if (rcode != PS_OK) return rcode;
+  }
+  if (dW) {
+    CUtensorMap ta, tb;
+    if (!map_mnmajor(&ta, dz, rc, V, ldz) || !map_mnmajor(&tb, Hpk, rc, d, d)) return PS_ERR_INVALID_ARG;
+    StoreF32Epi::Params ep{dW, d, V, d, dw_accumulate};
+    rcode = launch_gemm<true, true, StoreF32Epi>(ta, tb, V, d, rc, 0, 16, ep, status, s);
+    if (rcode != PS_OK) return rcode;
+  }
+  return PS_OK;
+}
+
+int gemm_bf16(int M, int N, int K, int a_mn, int b_mn, const void* A, int64_t lda, const void* B, int64_t ldb,
+              float* C, int64_t ldc, int accumulate, uint32_t* status, cudaStream_t s) {
+  CUtensorMap ta, tb;
+  const bool oka = a_mn ? map_mnmajor(&ta, A, K, M, lda) : map_kmajor(&ta, A, M, K, lda, kBM);
+  const bool okb = b_mn ? map_mnmajor(&tb, B, K, N, ldb) : map_kmajor(&tb, B, N, K, ldb, kBN);
+  if (!oka || !okb) return PS_ERR_INVALID_ARG;
+  StoreF32Epi::Params ep{C, ldc, M, N, accumulate};
+  if (!a_mn && !b_mn) return launch_gemm<false, false, StoreF32Epi>(ta, tb, M, N, K, 0, 16, ep, status, s);
+  if (!a_mn && b_mn) return launch_gemm<false, true, StoreF32Epi>(ta, tb, M, N, K, 0, 16, ep, status, s);
+  if (a_mn && b_mn) return launch_gemm<true, true, StoreF32Epi>(ta, tb, M, N, K, 0, 16, ep, status, s);
+  return launch_gemm<true, false, StoreF32Epi>(ta, tb, M, N, K, 0, 16, ep, status, s);
+}
+
+// ----------------------------------------------------------------------------- wait probe
+__global__ void wait_probe_kernel(uint64_t timeout_ns, uint32_t* status) {
+  __shared__ uint64_t bar;
+  if (threadIdx.x == 0) {
+    mbar_init(&bar, 1);
+    fence_mbar_init();
+  }
+  __syncthreads();
+  if (threadIdx.x == 0 && !mbar_wait(&bar, 0, timeout_ns, nullptr)) raise_status(status, PS_DEV_TIMEOUT);
+}
+
+int wait_timeout_probe(uint64_t timeout_ns, uint32_t* status, cudaStream_t s) {
+  wait_probe_kernel<<<1, 32, 0, s>>>(timeout_ns, status);
+  return cudaGetLastError() == cudaSuccess ? PS_OK : PS_ERR_CUDA;
+}
+
+}  // namespace psk

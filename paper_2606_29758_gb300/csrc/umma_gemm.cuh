@@ -1,0 +1,244 @@
+// Persistent, warp-specialised tcgen05 GEMM for sm_103a with pluggable epilogues.
+//
+//   D[M, N] = sum_k A[m, k] B[n, k]      (bf16 operands, f32 accumulation in TMEM)
+//
+// A is K-major ([M][K] in memory) or MN-major ([K][M]); likewise B ([N][K] or [K][N]).
+// Tiles of 128 x 256 outputs, 64-deep K blocks, 4-stage shared-memory ring fed by TMA
+// with 128-byte swizzle. Roles (192 threads):
+//   warp 0      TMA producer (one lane)
+//   warp 1      TMEM allocator + MMA issuer (one lane)
+//   warps 2..5  epilogue: each thread owns one accumulator row (TMEM lane) and reads
+//               its 256 columns in chunks of 32 with tcgen05.ld
+// Two 256-column accumulators (all 512 TMEM columns) let the epilogue of one tile
+// overlap the main loop of the next. Every wait is bounded; on expiry the kernel sets
+// PS_DEV_TIMEOUT, waits (bounded) for its own loads in flight, frees TMEM and returns.
+//
+// Work is split into units: unit u is (m block, range of n blocks [n0, n1)), walked in
+// order by one CTA, so an epilogue can keep per-row state across a unit's tiles (the
+// forward's running logsumexp). Units are enumerated in bands of `band_m` m-blocks;
+// inside a band the split index is the slow coordinate, so CTAs that run at the same
+// time share B panels (and A panels) through L2.
+#pragma once
+
+#include "ps_common.cuh"
+
+namespace psk {
+
+constexpr int kBM = 128;
+constexpr int kBN = 256;
+constexpr int kBK = 64;
+constexpr int kStages = 4;
+constexpr int kGemmThreads = 192;
+constexpr int kEpiWarp0 = 2;
+constexpr uint32_t kTileABytes = kBM * kBK * 2;   // 16 KB
+constexpr uint32_t kTileBBytes = kBN * kBK * 2;   // 32 KB
+constexpr uint32_t kTmemCols = 512;               // two 256-column f32 accumulators
+
+struct Sched {
+  int m_blocks;   // ceil(M / 128)
+  int n_blocks;   // ceil(N / 256)
+  int splits;     // n-ranges per m block (n_blocks: one tile per unit)
+  int band_m;     // m blocks per band
+  int num_units;  // m_blocks * splits
+  int num_kb;     // ceil(K / 64)
+
+  __device__ __forceinline__ void unit(int u, int& m_blk, int& split, int& n0, int& n1) const {
+    const int per_band = band_m * splits;
+    const int band = u / per_band;
+    const int r = u - band * per_band;
+    const int m_first = band * band_m;
+    const int this_band = min(band_m, m_blocks - m_first);
+    split = r / this_band;
+    m_blk = m_first + (r - split * this_band);
+    n0 = static_cast<int>((static_cast<long long>(split) * n_blocks) / splits);
+    n1 = static_cast<int>((static_cast<long long>(split + 1) * n_blocks) / splits);
+  }
+};
+
+struct GemmSmem {
+  // 1024-byte aligned tile ring first (128-byte swizzle atoms repeat every 1 KB)
+  uint8_t a[kStages][kTileABytes];
+  uint8_t b[kStages][kTileBBytes];
+  uint64_t full[kStages];
+  uint64_t empty[kStages];
+  uint64_t tfull[2];
+  uint64_t tempty[2];
+  uint64_t drain;
+  uint32_t tmem_base;
+  int abort;
+};
+constexpr size_t kGemmSmemBytes = sizeof(GemmSmem) + 1024;  // + alignment slack
+
+template <bool A_MN, bool B_MN, class Epi>
+__global__ void __launch_bounds__(kGemmThreads, 1)
+    umma_gemm_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmB,
+                     const Sched sched, const typename Epi::Params ep, uint32_t* status, uint64_t timeout_ns) {
+  extern __shared__ uint8_t smem_raw[];
+  GemmSmem& sm = *reinterpret_cast<GemmSmem*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
+  const int warp = threadIdx.x >> 5;
+  const int lane = threadIdx.x & 31;
+
+  if (threadIdx.x == 0) {
+    for (int s = 0; s < kStages; ++s) {
+      mbar_init(&sm.full[s], 1);
+      mbar_init(&sm.empty[s], 1);
+    }
+    for (int a = 0; a < 2; ++a) {
+      mbar_init(&sm.tfull[a], 1);
+      mbar_init(&sm.tempty[a], 128);
+    }
+    mbar_init(&sm.drain, 1);
+    sm.abort = 0;
+    fence_mbar_init();
+  }
+  if (warp == 0 && lane == 0) {
+    tma_prefetch_desc(&tmA);
+    tma_prefetch_desc(&tmB);
+  }
+  if (warp == 1) {
+    tmem_alloc(&sm.tmem_base, kTmemCols);
+    tmem_relinquish();
+  }
+  tc_fence_before();
+  __syncthreads();
+  tc_fence_after();
+  const uint32_t tmem_base = sm.tmem_base;
+  volatile int* abort = &sm.abort;
+
+  if (warp == 0) {
+    // ------------------------------------------------------------------ TMA producer
+    if (lane == 0) {
+      uint32_t kc = 0;  // k blocks issued by this CTA
+      bool ok = true;
+      for (int u = blockIdx.x; ok && u < sched.num_units; u += gridDim.x) {
+        int m_blk, split, n0, n1;
+        sched.unit(u, m_blk, split, n0, n1);
+        for (int nb = n0; ok && nb < n1; ++nb) {
+          for (int kb = 0; kb < sched.num_kb; ++kb, ++kc) {
+            const int s = kc % kStages;
+            const uint32_t ph = (kc / kStages) & 1u;
+            if (!mbar_wait(&sm.empty[s], ph ^ 1u, timeout_ns, abort)) { ok = false; break; }
+            mbar_arrive_expect_tx(&sm.full[s], kTileABytes + kTileBBytes);
+            const int m0 = m_blk * kBM, nn0 = nb * kBN, k0 = kb * kBK;
+            if (A_MN) {
+              for (int i = 0; i < kBM / 64; ++i)
+                tma_load_2d(sm.a[s] + i * (kBK * 128), &tmA, &sm.full[s], m0 + i * 64, k0);
+            } else {
+              tma_load_2d(sm.a[s], &tmA, &sm.full[s], k0, m0);
+            }
+            if (B_MN) {
+              for (int i = 0; i < kBN / 64; ++i)
+                tma_load_2d(sm.b[s] + i * (kBK * 128), &tmB, &sm.full[s], nn0 + i * 64, k0);
+            } else {
+              tma_load_2d(sm.b[s], &tmB, &sm.full[s], k0, nn0);
+            }
+          }
+        }
+      }
+      if (!ok) {
+        *abort = 1;
+        raise_status(status, PS_DEV_TIMEOUT);
+        // let the loads already issued land before the CTA can exit
+        const uint32_t first = kc > kStages ? kc - kStages : 0;
+        for (uint32_t j = first; j < kc; ++j)
+          mbar_wait(&sm.full[j % kStages], (j / kStages) & 1u, timeout_ns, nullptr);
+      }
+    }
+  } else if (warp == 1) {
+    // ------------------------------------------------------------------ MMA issuer
+    if (lane == 0) {
+      constexpr uint32_t idesc = idesc_bf16_f32(kBM, kBN, A_MN, B_MN);
+      // K-major: 8-row groups 1024 B apart; a 16-deep K step is 32 B inside the swizzle atom.
+      // MN-major: 64-element atoms kBK*128 B apart (LBO); 8-row K groups 1024 B apart (SBO);
+      //           a 16-deep K step is 16 rows = 2048 B.
+      constexpr uint32_t a_lbo = A_MN ? kBK * 128 : 16, a_step = A_MN ? 2048 : 32;
+      constexpr uint32_t b_lbo = B_MN ? kBK * 128 : 16, b_step = B_MN ? 2048 : 32;
+      uint32_t kc = 0, tile = 0;
+      bool ok = true;
+      for (int u = blockIdx.x; ok && u < sched.num_units; u += gridDim.x) {
+        int m_blk, split, n0, n1;
+        sched.unit(u, m_blk, split, n0, n1);
+        for (int nb = n0; ok && nb < n1; ++nb, ++tile) {
+          const uint32_t acc = tile & 1u;
+          const uint32_t aph = (tile >> 1) & 1u;
+          if (!mbar_wait(&sm.tempty[acc], aph ^ 1u, timeout_ns, abort)) { ok = false; break; }
+          tc_fence_after();
+          const uint32_t d_tmem = tmem_base + acc * kBN;
+          for (int kb = 0; kb < sched.num_kb; ++kb, ++kc) {
+            const int s = kc % kStages;
+            const uint32_t ph = (kc / kStages) & 1u;
+            if (!mbar_wait(&sm.full[s], ph, timeout_ns, abort)) { ok = false; break; }
+            tc_fence_after();
+            const uint32_t a_base = smem_addr(sm.a[s]);
+            const uint32_t b_base = smem_addr(sm.b[s]);
+#pragma unroll
+            for (int k = 0; k < kBK / 16; ++k) {
+              const uint64_t ad = smem_desc_sw128(a_base + k * a_step, a_lbo, 1024);
+              const uint64_t bd = smem_desc_sw128(b_base + k * b_step, b_lbo, 1024);
+              umma_bf16(d_tmem, ad, bd, idesc, (kb | k) != 0 ? 1u : 0u);
+            }
+            umma_commit(&sm.empty[s]);  // frees the stage once these MMAs have read it
+          }
+          if (ok) umma_commit(&sm.tfull[acc]);  // accumulator ready for the epilogue
+        }
+      }
+      if (!ok) {
+        *abort = 1;
+        raise_status(status, PS_DEV_TIMEOUT);
+        // wait (bounded) until the MMAs already issued have finished with TMEM
+        umma_commit(&sm.drain);
+        mbar_wait(&sm.drain, 0, timeout_ns, nullptr);
+      }
+    }
+  } else {
+    // ------------------------------------------------------------------ epilogue
+    const int quad = warp & 3;                  // TMEM lanes 32*quad .. 32*quad+31
+    const int row_in_tile = quad * 32 + lane;
+    typename Epi::State st;
+    uint32_t tile = 0;
+    bool ok = true;
+    for (int u = blockIdx.x; ok && u < sched.num_units; u += gridDim.x) {
+      int m_blk, split, n0, n1;
+      sched.unit(u, m_blk, split, n0, n1);
+      const int row = m_blk * kBM + row_in_tile;
+      Epi::begin_unit(ep, st, row, split);
+      for (int nb = n0; nb < n1; ++nb, ++tile) {
+        const uint32_t acc = tile & 1u;
+        const uint32_t aph = (tile >> 1) & 1u;
+        // one lane waits; the warp follows it, so tcgen05.ld always runs on a converged warp
+        int got = 0;
+        if (lane == 0) got = mbar_wait(&sm.tfull[acc], aph, timeout_ns, abort) ? 1 : 0;
+        got = __shfl_sync(0xffffffffu, got, 0);
+        if (!got) { ok = false; break; }
+        tc_fence_after();
+        const uint32_t t_row = tmem_base + (static_cast<uint32_t>(quad * 32) << 16) + acc * kBN;
+#pragma unroll 1
+        for (int c = 0; c < kBN / 32; ++c) {
+          uint32_t r[32];
+          tmem_ld32(t_row + c * 32, r);
+          tmem_ld_wait();
+          if (c == kBN / 32 - 1) {
+            // the accumulator has been read completely: hand it back to the MMA warp
+            tc_fence_before();
+            mbar_arrive(&sm.tempty[acc]);
+          }
+          Epi::chunk(ep, st, row, nb * kBN + c * 32, r);
+        }
+      }
+      if (ok) Epi::end_unit(ep, st, row, split);
+    }
+    if (!ok) {
+      *abort = 1;
+      raise_status(status, PS_DEV_TIMEOUT);
+    }
+  }
+
+  tc_fence_before();
+  __syncthreads();
+  if (warp == 1) {
+    tc_fence_after();
+    tmem_dealloc(tmem_base, kTmemCols);
+  }
+}
+
+}  // namespace psk

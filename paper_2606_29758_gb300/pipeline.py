@@ -1,0 +1,106 @@
+"""One PS-PPO LM-head update pass through the C ABI, with buffers held in torch.
+
+UpdatePass owns the device buffers of one batch shape (allocated once with torch,
+sized for the worst case N = sum L) and runs the four library calls in order on the
+current stream: cutoffs -> packed prefixes -> fused forward -> fused backward.
+The only host synchronisation is reading N after packing.
+"""
+from __future__ import annotations
+
+from dataclasses import dataclass
+from typing import Optional
+
+import torch
+
+from . import _binding as B
+
+
+@dataclass
+class PassShape:
+    P: int
+    K: int
+    T_max: int
+    d: int
+    V: int
+    capacity: int                 # max packed rows (sum of lengths)
+    dtype: torch.dtype = torch.bfloat16
+    bwd_chunk_rows: int = 32768   # rows of dZ held at once in the backward workspace
+
+
+class UpdatePass:
+    def __init__(self, shape: PassShape, device: str = "cuda", eps: float = 0.2, loss_scale: Optional[float] = None,
+                 mode: int = B.PS_MODE_TRUNC, adv_mode: int = B.PS_ADV_GROUP_NORM):
+        s = shape
+        self.s, self.device, self.eps, self.mode, self.adv_mode = s, device, eps, mode, adv_mode
+        self.loss_scale = loss_scale if loss_scale is not None else 1.0 / (s.P * s.K)
+        self.dcode = B.dtype_code(torch.empty(0, dtype=s.dtype))
+        Bn, cap = s.P * s.K, s.capacity
+        i32 = dict(dtype=torch.int32, device=device)
+        f32 = dict(dtype=torch.float32, device=device)
+        self.H = torch.empty(Bn, **i32)
+        self.n = torch.empty(Bn, **i32)
+        self.w_tab = torch.empty(s.P, s.T_max, **f32)
+        self.cu_seqlens = torch.empty(Bn + 1, **i32)
+        self.src_row = torch.empty(cap, **i32)
+        self.row_traj = torch.empty(cap, **i32)
+        self.row_pos = torch.empty(cap, **i32)
+        self.tok = torch.empty(cap, **i32)
+        self.oldlogp = torch.empty(cap, **f32)
+        self.w = torch.empty(cap, **f32)
+        self.adv = torch.empty(cap, **f32)
+        self.hid = torch.empty(cap, s.d, dtype=s.dtype, device=device)
+        self.lse = torch.empty(cap, **f32)
+        self.logp = torch.empty(cap, **f32)
+        self.ratio = torch.empty(cap, **f32)
+        self.coef = torch.empty(cap, **f32)
+        self.row_loss = torch.empty(cap, **f32)
+        self.loss = torch.zeros(1, dtype=torch.float64, device=device)
+        self.dH = torch.empty(cap, s.d, **f32)
+        self.dW = torch.empty(s.V, s.d, **f32)
+        u8 = dict(dtype=torch.uint8, device=device)
+        self.ws_samp = torch.empty(B.ps_sample_cutoffs_workspace_size(s.P, s.K, s.T_max), **u8)
+        self.ws_pack = torch.empty(B.ps_pack_prefixes_workspace_size(s.P, s.K), **u8)
+        self.ws_fwd = torch.empty(B.ps_lmhead_ppo_fwd_workspace_size(cap, s.d, s.V, self.dcode), **u8)
+        self.ws_bwd = torch.empty(B.ps_lmhead_ppo_bwd_workspace_size(cap, s.d, s.V, self.dcode,
+                                                                     min(s.bwd_chunk_rows, cap)), **u8)
+        self.N = 0
+
+    def sample(self, q, L, seed, step, traj_base=0):
+        s = self.s
+        B.ps_sample_cutoffs(s.P, s.K, s.T_max, q, L, seed, step, traj_base, self.mode, self.H, self.n,
+                            self.w_tab, self.ws_samp)
+
+    def pack(self, L, R, tok_full, oldlogp_full, hid_full) -> int:
+        s = self.s
+        self.N = B.ps_pack_prefixes(s.P, s.K, s.T_max, s.d, self.dcode, L, self.n, R, self.adv_mode, self.w_tab,
+                                    tok_full, oldlogp_full, hid_full, s.capacity, self.cu_seqlens, self.src_row,
+                                    self.row_traj, self.row_pos, self.tok, self.oldlogp, self.w, self.adv, self.hid,
+                                    self.ws_pack)
+        return self.N
+
+    def forward(self, W):
+        s = self.s
+        B.ps_lmhead_ppo_fwd(self.N, s.d, s.V, self.dcode, self.hid, W, self.tok, self.oldlogp, self.adv, self.w,
+                            self.eps, self.loss_scale, self.loss, self.lse, self.logp, self.ratio, self.coef,
+                            self.row_loss, self.ws_fwd)
+
+    def backward(self, W, dw_accumulate: bool = False):
+        s = self.s
+        B.ps_lmhead_ppo_bwd(self.N, s.d, s.V, self.dcode, self.hid, W, self.tok, self.lse, self.coef, self.dH,
+                            self.dW, B.PS_DW_ACCUMULATE if dw_accumulate else B.PS_DW_OVERWRITE, self.ws_bwd)
+
+    def run(self, q, L, R, tok_full, oldlogp_full, hid_full, W, seed, step, traj_base=0, grads=True) -> int:
+        self.sample(q, L, seed, step, traj_base)
+        self.pack(L, R, tok_full, oldlogp_full, hid_full)
+        self.forward(W)
+        if grads:
+            self.backward(W)
+        return self.N
+
+    def check_status(self):
+        """Raise PsppoError if any workspace reports a device-side error."""
+        for name, ws in (("sample", self.ws_samp), ("pack", self.ws_pack), ("fwd", self.ws_fwd),
+                         ("bwd", self.ws_bwd)):
+            rc, bits = B.ps_workspace_status(ws)
+            if rc != B.PS_OK:
+                raise B.PsppoError(rc, f"{name} (device bits {bits:#x})")
