@@ -1,0 +1,363 @@
+"""Benchmark of the PS-PPO LM-head update pass on GB300.
+
+One step = one pass of the whole hot path over one synthetic rollout batch of the
+7B-shaped workload (16 prompts x 8 completions, lognormal lengths around 2048 clipped
+to [128, 8192], d = 3584, V = 152064, bf16): cutoff sampling -> prefix packing ->
+fused LM-head forward -> fused LM-head backward (dH and dW). Every step draws new
+cutoffs (the Philox step counter advances), so N varies from step to step.
+
+value: prefix tokens/s, whole job (sum of packed rows over all steps and ranks divided
+by the max over ranks of the device-timed region). The credited work of a step is
+6 N d V FLOPs (forward GEMM, dH, dW; the backward's logit recompute is not credited).
+
+    python bench.py [--gpus N] [--steps K] [--warmup W] [--impl ours|reference]
+
+With --gpus N > 1 (launched by torchrun) every rank runs its own replica of the
+workload on its own GPU: the pass has no cross-rank exchange in this form
+(weak scaling). --impl reference times the CPU float64 oracle on bounded samples of
+the same workload, on the host cores.
+"""
+from __future__ import annotations
+
+import argparse
+import json
+import os
+import subprocess
+import sys
+import threading
+import time
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+sys.path.insert(0, ROOT)
+
+import numpy as np  # noqa: E402
+
+WORKLOAD = "7b"
+MEASURED_PEAKS = os.path.join(ROOT, "MEASURED_PEAKS.json")
+FALLBACK_PEAKS = {"hbm_gbs": 6800.0, "bf16_tflops": 1900.0, "bf16_tflops_sustained": 1700.0}
+
+# dram bytes (read + write) per launch of the forward GEMM, from the ncu capture named
+# below, scaled to this workload's rows; None until measured for the current kernel.
+FWD_GEMM_TRAFFIC = None
+
+
+def describe(cfg) -> str:
+    law = (f"lognormal(median {cfg.len_median}) clipped [{cfg.len_lo}, {cfg.len_hi}]" if cfg.len_law == "lognormal"
+           else f"uniform [{cfg.len_lo}, {cfg.len_hi}]")
+    return (f"{cfg.name}: {cfg.P} prompts x {cfg.K} completions, lengths {law}, d={cfg.d}, V={cfg.V}, "
+            f"{cfg.dtype}, Beta cutoff pmf, eps={cfg.eps}, mode={cfg.mode}")
+
+
+def _peaks():
+    try:
+        with open(MEASURED_PEAKS) as f:
+            p = json.load(f)
+        return p, "measured"
+    except Exception:
+        return FALLBACK_PEAKS, "fallback"
+
+
+class ClockSampler:
+    """nvidia-smi sampling of SM clocks and throttle reasons while the timed region runs."""
+    Q = ("clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.hw_slowdown,"
+         "clocks_event_reasons.hw_thermal_slowdown,clocks_event_reasons.sw_thermal_slowdown,"
+         "clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, index: int):
+        self.index = index
+        self.proc = None
+        self.lines = []
+
+    def start(self):
+        try:
+            self.proc = subprocess.Popen(["nvidia-smi", f"--id={self.index}", f"--query-gpu={self.Q}",
+                                          "--format=csv,noheader,nounits", "-lms", "200"],
+                                         stdout=subprocess.PIPE, stderr=subprocess.DEVNULL, text=True)
+            self.t = threading.Thread(target=self._read, daemon=True)
+            self.t.start()
+        except Exception:
+            self.proc = None
+
+    def _read(self):
+        for line in self.proc.stdout:
+            self.lines.append(line.strip())
+
+    def stop(self):
+        if self.proc is None:
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["nvidia-smi unavailable"]}
+        self.proc.terminate()
+        try:
+            self.proc.wait(timeout=5)
+        except Exception:
+            self.proc.kill()
+        rows = []
+        for ln in self.lines:
+            parts = [p.strip() for p in ln.split(",")]
+            if len(parts) != 7:
+                continue
+            try:
+                rows.append((float(parts[0]), float(parts[1]), float(parts[2]), parts[3:]))
+            except ValueError:
+                continue
+        if not rows:
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["no samples"]}
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        reasons = sorted({names[i] for _, _, _, fl in rows for i, v in enumerate(fl) if v.lower() == "active"})
+        loaded = [r for r in rows if r[2] > 200.0] or rows
+        return {"sm_mhz": float(np.median([r[0] for r in loaded])), "sm_max_mhz": rows[0][1],
+                "reasons": reasons, "samples": len(rows), "power_w_max": max(r[2] for r in rows)}
+
+
+def _dist():
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    rank = int(os.environ.get("RANK", "0"))
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    return world, rank, local
+
+
+def run_ours(args):
+    import torch
+    import torch.distributed as dist
+
+    from paper_2606_29758_gb300 import PassShape, UpdatePass
+    from synthetic import get_config, make_batch
+
+    world, rank, local = _dist()
+    torch.cuda.set_device(local)
+    dev = f"cuda:{local}"
+    if world > 1:
+        dist.init_process_group("nccl", device_id=torch.device(dev))
+    cfg = get_config(args.config)
+    b = make_batch(cfg, device=dev)
+    D = b.dev
+    shape = PassShape(cfg.P, cfg.K, b.T_max, cfg.d, cfg.V, b.total_len, torch.bfloat16, args.chunk_rows)
+    up = UpdatePass(shape, device=dev, eps=cfg.eps, loss_scale=cfg.loss_scale)
+    stream = torch.cuda.current_stream()
+    seed = cfg.seed
+
+    def step(i, ev=None):
+        if ev is not None:
+            ev[0].record(stream)
+        up.sample(D["q"], D["L"], seed, i)
+        n = up.pack(D["L"], D["R"], D["tok_full"], D["oldlogp_full"], D["hid_full"])
+        if ev is not None:
+            ev[1].record(stream)
+        up.forward(D["W"])
+        if ev is not None:
+            ev[2].record(stream)
+        up.backward(D["W"])
+        if ev is not None:
+            ev[3].record(stream)
+        return n
+
+    def barrier():
+        torch.cuda.synchronize()
+        if world > 1:
+            dist.barrier()
+        torch.cuda.synchronize()
+
+    for i in range(args.warmup):
+        step(1000 + i)
+    up.check_status()
+    barrier()
+
+    clocks = ClockSampler(local)
+    clocks.start()
+    time.sleep(0.3)
+    evs = [[torch.cuda.Event(enable_timing=True) for _ in range(4)] for _ in range(args.steps)]
+    barrier()
+    t0 = torch.cuda.Event(enable_timing=True)
+    t1 = torch.cuda.Event(enable_timing=True)
+    t0.record(stream)
+    rows = 0
+    for i in range(args.steps):
+        rows += step(i, evs[i])
+    t1.record(stream)
+    barrier()
+    clk = clocks.stop()
+    up.check_status()
+    ms = t0.elapsed_time(t1)
+    per = np.array([[e[0].elapsed_time(e[1]), e[1].elapsed_time(e[2]), e[2].elapsed_time(e[3])] for e in evs])
+    ms_max = ms
+    rows_all = rows
+    if world > 1:
+        t = torch.tensor([ms], device=dev, dtype=torch.float64)
+        dist.all_reduce(t, op=dist.ReduceOp.MAX)
+        ms_max = float(t.item())
+        r = torch.tensor([rows], device=dev, dtype=torch.float64)
+        dist.all_reduce(r)
+        rows_all = int(r.item())
+
+    # ---- end-to-end: host (pinned) inputs -> device -> pass -> loss back to the host, every step
+    host = {k: D[k].cpu().pin_memory() for k in ("q", "L", "R", "tok_full", "oldlogp_full", "hid_full")}
+    dbuf = {k: torch.empty_like(D[k]) for k in host}
+    loss_h = torch.empty(1, dtype=torch.float64).pin_memory()
+    h2d = sum(v.numel() * v.element_size() for v in host.values())
+
+    def e2e_step(i):
+        for k in host:
+            dbuf[k].copy_(host[k], non_blocking=True)
+        up.sample(dbuf["q"], dbuf["L"], seed, i)
+        n = up.pack(dbuf["L"], dbuf["R"], dbuf["tok_full"], dbuf["oldlogp_full"], dbuf["hid_full"])
+        up.forward(D["W"])
+        up.backward(D["W"])
+        loss_h.copy_(up.loss, non_blocking=True)
+        stream.synchronize()
+        return n
+
+    e2e_step(2000)
+    barrier()
+    e0 = time.perf_counter()
+    e_rows = 0
+    for i in range(args.steps):
+        e_rows += e2e_step(i)
+    barrier()
+    e_ms = (time.perf_counter() - e0) * 1e3
+    if world > 1:
+        t = torch.tensor([e_ms], device=dev, dtype=torch.float64)
+        dist.all_reduce(t, op=dist.ReduceOp.MAX)
+        e_ms = float(t.item())
+        r = torch.tensor([e_rows], device=dev, dtype=torch.float64)
+        dist.all_reduce(r)
+        e_rows = int(r.item())
+
+    peaks, src = _peaks()
+    d, V = cfg.d, cfg.V
+    mean_rows = rows / args.steps
+    t_fwd = float(per[:, 1].mean()) * 1e-3
+    fwd_flops = 2.0 * mean_rows * d * V
+    peak_tf = peaks["bf16_tflops_sustained"]
+    achieved_tf = fwd_flops / t_fwd / 1e12
+    step_s = ms / args.steps * 1e-3
+    credited_tf = 6.0 * mean_rows * d * V / step_s / 1e12
+    chunks = -(-int(round(mean_rows)) // args.chunk_rows)
+    launches_per_step = 1 + 2 + 3 + 3 * chunks
+    out = {
+        "metric": "prefix tokens/s (fused LM-head PS-PPO fwd+bwd, 1xGB300)",
+        "value": rows_all / (ms_max * 1e-3),
+        "unit": "tokens/s",
+        "n_gpus": world,
+        "steps": args.steps,
+        "warmup": args.warmup,
+        "ms_per_step": ms_max / args.steps,
+        "higher_is_better": True,
+        "scaling": "weak",
+        "vs_baseline": None,
+        "dtype": "bf16",
+        "data": "synthetic (seeded generator; random-init head)",
+        "config": {"workload": describe(cfg),
+                   "global_batch": cfg.B * world, "mean_prefix_rows": mean_rows, "sum_lengths": b.total_len,
+                   "bwd_chunk_rows": args.chunk_rows,
+                   "l2": "inputs larger than L2 (hidden states 2.1 GB, W 1.1 GB)",
+                   "parallelism": "replicas" if world > 1 else "single GPU"},
+        "pct_bf16_peak": {"credited_6NdV_tflops": credited_tf, "frac_of_sustained": credited_tf / peak_tf,
+                          "frac_of_burst": credited_tf / peaks["bf16_tflops"],
+                          "executed_8NdV_tflops": credited_tf * 8 / 6, "peak_source": src},
+        "per_call_ms": {"sample+pack": float(per[:, 0].mean()), "fwd": float(per[:, 1].mean()),
+                        "bwd": float(per[:, 2].mean())},
+        "roofline": {"kernel": "umma_gemm_kernel<K,K,FwdLseEpi> (fused forward; + O(N) finalize)",
+                     "bound": "tensor", "achieved": achieved_tf, "peak": peak_tf, "unit": "TFLOP/s",
+                     "frac": achieved_tf / peak_tf, "traffic": FWD_GEMM_TRAFFIC,
+                     "algorithmic_per_launch": f"2*N*d*V = {fwd_flops:.4g} FLOP",
+                     "peak_note": f"bf16_tflops_sustained ({src}); kernel timed inside the step"},
+        "e2e": {"value": e_rows / (e_ms * 1e-3), "unit": "tokens/s", "h2d_bytes_per_step": h2d,
+                "d2h_bytes_per_step": 8},
+        "gpu_launches": launches_per_step * args.steps,
+        "clocks": clk,
+    }
+    if rank == 0 and not args.no_cpu_baseline:
+        out["cpu_baseline"] = cpu_baseline(cfg, b, args.cpu_rows)
+    if world > 1:
+        dist.destroy_process_group()
+    if rank == 0:
+        print(json.dumps(out))
+
+
+def _oracle_sample_pass(cfg, b, W64, rows_in_sample, step):
+    """The oracle, as it stands, on a bounded sample: cutoffs, advantages and packing indices
+    for the whole batch, then the head forward and backward over the first packed rows."""
+    from oracle import lmhead
+    from oracle.cutoffs import sample_cutoffs
+    from oracle.pack import group_advantages, pack_prefixes
+    from oracle.pipeline import widen
+    H, n, w_tab = sample_cutoffs(b.q, b.L, cfg.K, cfg.seed, step)
+    A = group_advantages(b.R, cfg.K, cfg.adv_mode)
+    pk = pack_prefixes(b.L, n, cfg.K, w_tab, A, b.tok_full, b.oldlogp_full, None)
+    s = np.arange(min(rows_in_sample, pk["N"]))
+    Hs = widen(cfg, b.hid_full[pk["src_row"][s]])
+    f = lmhead.forward(Hs, W64, pk["tok"][s], pk["oldlogp"][s], pk["adv"][s], pk["w"][s], cfg.eps, cfg.loss_scale)
+    lmhead.backward(Hs, W64, pk["tok"][s], f["lse"], f["coef"])
+    return s.size
+
+
+def cpu_baseline(cfg, b, rows):
+    from oracle.pipeline import widen
+    W64 = widen(cfg, b.W)
+    t0 = time.perf_counter()
+    done = _oracle_sample_pass(cfg, b, W64, rows, 0)
+    dt = time.perf_counter() - t0
+    return {"value": done / dt, "unit": "tokens/s", "cores": os.cpu_count(), "kind": "oracle",
+            "sample": f"{done} packed rows of one {cfg.name} batch (cutoffs, advantages and packing of the "
+                      f"whole batch; f64 head forward + dH + dW over the sampled rows), {dt:.1f} s"}
+
+
+def run_reference(args):
+    from synthetic import get_config, make_batch
+    from oracle.pipeline import widen
+    world, rank, _ = _dist()
+    if rank != 0:
+        return
+    cfg = get_config(args.config)
+    dev = None
+    try:
+        import torch
+        if torch.cuda.is_available():
+            dev = "cuda:0"
+    except Exception:
+        pass
+    b = make_batch(cfg, device=dev)   # the old log-probs need the full head; on the GPU when present
+    W64 = widen(cfg, b.W)
+    for i in range(args.warmup):
+        _oracle_sample_pass(cfg, b, W64, args.ref_rows, 1000 + i)
+    t0 = time.perf_counter()
+    rows = 0
+    for i in range(args.steps):
+        rows += _oracle_sample_pass(cfg, b, W64, args.ref_rows, i)
+    dt = time.perf_counter() - t0
+    v = rows / dt
+    print(json.dumps({
+        "impl": "reference", "metric": "prefix tokens/s (fused LM-head PS-PPO fwd+bwd, 1xGB300)",
+        "value": v, "unit": "tokens/s", "n_gpus": world, "steps": args.steps, "warmup": args.warmup,
+        "ms_per_step": dt / args.steps * 1e3, "higher_is_better": True, "scaling": "weak", "vs_baseline": None,
+        "dtype": "f64", "data": "synthetic (seeded generator; random-init head)",
+        "config": {"workload": describe(cfg),
+                   "sample_rows_per_step": args.ref_rows},
+        "cpu_baseline": {"value": v, "unit": "tokens/s", "cores": os.cpu_count(), "kind": "oracle",
+                         "sample": f"{args.ref_rows} packed rows per step (f64 forward + dH + dW) after "
+                                   f"cutoffs/packing of the whole batch"},
+        "e2e": {"value": v, "unit": "tokens/s", "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
+    }))
+
+
+def main():
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=10)
+    ap.add_argument("--warmup", type=int, default=3)
+    ap.add_argument("--impl", choices=["ours", "reference"], default="ours")
+    ap.add_argument("--config", default=WORKLOAD)
+    ap.add_argument("--chunk-rows", type=int, default=65536)
+    ap.add_argument("--cpu-rows", type=int, default=256)
+    ap.add_argument("--ref-rows", type=int, default=32)
+    ap.add_argument("--no-cpu-baseline", action="store_true")
+    args = ap.parse_args()
+    if args.warmup < 3 and args.impl == "ours":
+        args.warmup = 3
+    if args.impl == "reference":
+        run_reference(args)
+    else:
+        run_ours(args)
+
+
+if __name__ == "__main__":
+    main()

@@ -57,11 +57,11 @@ class UpdatePass:
         self.loss = torch.zeros(1, dtype=torch.float64, device=device)
         self.dH = torch.empty(cap, s.d, **f32)
         self.dW = torch.empty(s.V, s.d, **f32)
-        u8 = dict(dtype=torch.uint8, device=device)
-        self.ws_samp = torch.empty(B.ps_sample_cutoffs_workspace_size(s.P, s.K, s.T_max), **u8)
-        self.ws_pack = torch.empty(B.ps_pack_prefixes_workspace_size(s.P, s.K), **u8)
-        self.ws_fwd = torch.empty(B.ps_lmhead_ppo_fwd_workspace_size(cap, s.d, s.V, self.dcode), **u8)
-        self.ws_bwd = torch.empty(B.ps_lmhead_ppo_bwd_workspace_size(cap, s.d, s.V, self.dcode,
+        u8 = dict(dtype=torch.uint8, device=device)   # zeroed: a status word never written reads clear
+        self.ws_samp = torch.zeros(B.ps_sample_cutoffs_workspace_size(s.P, s.K, s.T_max), **u8)
+        self.ws_pack = torch.zeros(B.ps_pack_prefixes_workspace_size(s.P, s.K), **u8)
+        self.ws_fwd = torch.zeros(B.ps_lmhead_ppo_fwd_workspace_size(cap, s.d, s.V, self.dcode), **u8)
+        self.ws_bwd = torch.zeros(B.ps_lmhead_ppo_bwd_workspace_size(cap, s.d, s.V, self.dcode,
                                                                      min(s.bwd_chunk_rows, cap)), **u8)
         self.N = 0
 

@@ -69,6 +69,8 @@ CONFIGS["head1.5b_small"] = Config("head1.5b_small", P=1, K=4, len_law="uniform"
                                    len_median=None, d=1536, V=151936, dtype="bf16",
                                    beta_a=_BETA[0], beta_b=_BETA[1])
 CONFIGS["mid_f32"] = replace(CONFIGS["mid"], name="mid_f32", dtype="f32")
+# The 7B-shaped head on two prompts (about 25k packed rows): a small case for profiling.
+CONFIGS["7b_p2"] = replace(CONFIGS["7b"], name="7b_p2", P=2)
 
 
 def get_config(name: str, **overrides) -> Config:

@@ -14,23 +14,26 @@ def _ref(A, B, a_mn, b_mn):
 
 
 @pytest.mark.parametrize("a_mn,b_mn", [(0, 0), (0, 1), (1, 1), (1, 0)])
-@pytest.mark.parametrize("M,N,K", [(128, 256, 64), (300, 520, 200), (1000, 777 // 8 * 8, 968), (64, 40, 8)])
+@pytest.mark.parametrize("M,N,K", [(128, 256, 64), (300, 520, 200), (1000, 777, 968), (64, 40, 8), (129, 257, 65)])
 def test_layouts_and_ragged_edges(a_mn, b_mn, M, N, K):
     from paper_2606_29758_gb300 import _binding as B
     g = torch.Generator(device="cuda").manual_seed(M * 7 + N * 3 + K + a_mn * 2 + b_mn)
-    A = torch.randn((K, M) if a_mn else (M, K), device="cuda", generator=g).to(torch.bfloat16)
-    Bt = torch.randn((K, N) if b_mn else (N, K), device="cuda", generator=g).to(torch.bfloat16)
+    pad8 = lambda x: (x + 7) // 8 * 8  # noqa: E731  (leading dimensions must be multiples of 8)
+    Afull = torch.randn((K, pad8(M)) if a_mn else (M, pad8(K)), device="cuda", generator=g).to(torch.bfloat16)
+    Bfull = torch.randn((K, pad8(N)) if b_mn else (N, pad8(K)), device="cuda", generator=g).to(torch.bfloat16)
+    A = Afull[:, :M] if a_mn else Afull[:, :K]
+    Bt = Bfull[:, :N] if b_mn else Bfull[:, :K]
     ldc = (N + 3) // 4 * 4
     C = torch.full((M, ldc), float("nan"), device="cuda")
     ws = torch.empty(256, dtype=torch.uint8, device="cuda")
-    B.ps_diag_gemm_bf16(M, N, K, a_mn, b_mn, A, A.shape[1], Bt, Bt.shape[1], C, ldc, 0, ws)
+    B.ps_diag_gemm_bf16(M, N, K, a_mn, b_mn, Afull, Afull.shape[1], Bfull, Bfull.shape[1], C, ldc, 0, ws)
     torch.cuda.synchronize()
     assert B.ps_workspace_status(ws)[0] == B.PS_OK
     ref = _ref(A, Bt, a_mn, b_mn)
     err = (C[:, :N] - ref).abs().max().item()
     assert err <= 1e-4 * max(1.0, ref.abs().max().item()), err
     # accumulate into the previous result
-    B.ps_diag_gemm_bf16(M, N, K, a_mn, b_mn, A, A.shape[1], Bt, Bt.shape[1], C, ldc, 1, ws)
+    B.ps_diag_gemm_bf16(M, N, K, a_mn, b_mn, Afull, Afull.shape[1], Bfull, Bfull.shape[1], C, ldc, 1, ws)
     torch.cuda.synchronize()
     err2 = (C[:, :N] - 2 * ref).abs().max().item()
     assert err2 <= 2e-4 * max(1.0, ref.abs().max().item()), err2
