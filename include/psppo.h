@@ -179,6 +179,38 @@ int ps_lmhead_ppo_bwd(int64_t N, int d, int V, int dtype, const void* Hpk, const
                       float* dH, float* dW, int flags,
                       void* ws, size_t ws_bytes, ps_stream_t stream);
 
+/* ---------------------------------------------------------------------------
+ * ps_lmhead_ppo_fwd_noalloc -- ps_lmhead_ppo_fwd for callers that cannot allocate.
+ *
+ * The paper has no counterpart: this is a deployment variant of the forward above.
+ * Some callers cannot allocate device memory for a workspace -- a plugin inside a
+ * framework that owns the GPU's memory pool and forbids cudaMalloc, or a deployment
+ * whose device memory plan is fixed at start-up. This call computes exactly what
+ * ps_lmhead_ppo_fwd computes (same arguments and outputs, same kernels), but takes
+ * its scratch from a static 64 MiB device array inside the library instead of a
+ * caller workspace. It allocates nothing (no cudaMalloc, no cudaFree, no allocating
+ * library routine).
+ *  - Memory: every GPU that loads the library holds the 64 MiB array until the
+ *    process exits.
+ *  - Limit: the problem's workspace (ps_lmhead_ppo_fwd_workspace_size) must fit in
+ *    64 MiB: about N <= 508,000 packed rows for bf16; for f32, N * ceil(V/64) * 8
+ *    bytes must fit. Larger problems return PS_ERR_UNSUPPORTED and launch nothing.
+ *  - Set-up: the first call on each device looks up the array's device address
+ *    (cudaGetSymbolAddress) with that device current; make that first call before
+ *    any stream capture.
+ *  - Sharing: every call on a device uses the same array, which keeps the last call's
+ *    contents. Calls that overlap on the GPU (e.g. on two streams without ordering)
+ *    race on it; order them. Each call clears the status word it uses.
+ *  - Device-side errors (e.g. a token id outside [0, V)) are still detected, but no
+ *    workspace is returned to read them from; a bad token id shows as NaN in logp and
+ *    loss.
+ * ------------------------------------------------------------------------- */
+int ps_lmhead_ppo_fwd_noalloc(int64_t N, int d, int V, int dtype, const void* Hpk, const void* W,
+                              const int32_t* tok, const float* oldlogp, const float* adv, const float* w,
+                              double eps, double loss_scale,
+                              double* loss, float* lse, float* logp, float* ratio, float* coef,
+                              float* row_loss, ps_stream_t stream);
+
 #ifdef __cplusplus
 }
 #endif

@@ -28,7 +28,7 @@ EXPORTS = [
     "ps_pack_prefixes_workspace_size", "ps_pack_prefixes",
     "ps_lmhead_ppo_fwd_workspace_size", "ps_lmhead_ppo_fwd",
     "ps_lmhead_ppo_bwd_workspace_size", "ps_lmhead_ppo_bwd",
-    "ps_diag_gemm_bf16", "ps_diag_wait_timeout",
+    "ps_diag_gemm_bf16", "ps_diag_wait_timeout", "ps_lmhead_ppo_fwd_noalloc",
 ]
 
 
@@ -70,6 +70,8 @@ _SIGS = {
     "ps_lmhead_ppo_bwd": (_i32, [_i64, _i32, _i32, _i32, _vp, _vp, _vp, _vp, _vp, _vp, _vp, _i32, _vp, _sz, _vp]),
     "ps_diag_gemm_bf16": (_i32, [_i32, _i32, _i32, _i32, _i32, _vp, _i64, _vp, _i64, _vp, _i64, _i32, _vp, _sz, _vp]),
     "ps_diag_wait_timeout": (_i32, [_u64, _vp, _sz, _vp]),
+    "ps_lmhead_ppo_fwd_noalloc": (_i32, [_i64, _i32, _i32, _i32, _vp, _vp, _vp, _vp, _vp, _vp, _f64, _f64,
+                                         _vp, _vp, _vp, _vp, _vp, _vp, _vp]),
 }
 
 
@@ -177,6 +179,16 @@ def ps_lmhead_ppo_fwd(N, d, V, dtype, Hpk, W, tok, oldlogp, adv, w, eps, loss_sc
                                  float(eps), float(loss_scale), _ptr(loss), _ptr(lse), _ptr(logp), _ptr(ratio),
                                  _ptr(coef), _ptr(row_loss), _ptr(ws), _nbytes(ws), _stream(stream))
     _check(rc, "ps_lmhead_ppo_fwd")
+
+
+def ps_lmhead_ppo_fwd_noalloc(N, d, V, dtype, Hpk, W, tok, oldlogp, adv, w, eps, loss_scale, loss, lse, logp, ratio,
+                              coef, row_loss, stream=None):
+    """The forward with the library's static device scratch instead of a workspace, for
+    callers that cannot allocate device memory (see include/psppo.h)."""
+    rc = lib().ps_lmhead_ppo_fwd_noalloc(N, d, V, dtype, _ptr(Hpk), _ptr(W), _ptr(tok), _ptr(oldlogp), _ptr(adv),
+                                         _ptr(w), float(eps), float(loss_scale), _ptr(loss), _ptr(lse), _ptr(logp),
+                                         _ptr(ratio), _ptr(coef), _ptr(row_loss), _stream(stream))
+    _check(rc, "ps_lmhead_ppo_fwd_noalloc")
 
 
 def ps_lmhead_ppo_bwd_workspace_size(N: int, d: int, V: int, dtype: int, chunk_rows: int = 0) -> int:

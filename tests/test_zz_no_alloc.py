@@ -1,0 +1,59 @@
+"""The allocation-free forward (ps_lmhead_ppo_fwd_noalloc) against the workspace forward.
+
+Callers that cannot allocate device memory (a plugin inside a framework that owns the GPU's
+memory pool, a deployment with a fixed device memory plan) use the variant whose scratch is a
+static device array inside the library. It must give the same outputs as ps_lmhead_ppo_fwd,
+call after call (the array keeps the previous call's contents). This file is collected last.
+"""
+import pytest
+import torch
+
+from synthetic import get_config, make_batch
+
+pytestmark = pytest.mark.gpu
+
+OUTS = ("lse", "logp", "ratio", "coef", "row_loss")
+
+
+def _prepared(name):
+    from paper_2606_29758_gb300 import PassShape, UpdatePass
+    cfg = get_config(name)
+    b = make_batch(cfg, device="cuda")
+    dt = torch.bfloat16 if cfg.dtype == "bf16" else torch.float32
+    up = UpdatePass(PassShape(cfg.P, cfg.K, b.T_max, cfg.d, cfg.V, b.total_len, dt), eps=cfg.eps,
+                    loss_scale=cfg.loss_scale)
+    D = b.dev
+    up.sample(D["q"], D["L"], cfg.seed, cfg.step)
+    up.pack(D["L"], D["R"], D["tok_full"], D["oldlogp_full"], D["hid_full"])
+    up.forward(D["W"])              # the existing entry point, with a caller workspace
+    torch.cuda.synchronize()
+    up.check_status()
+    return cfg, D, up
+
+
+@pytest.mark.parametrize("name", ["mid", "head7b_small", "tiny"])
+def test_noalloc_forward_matches_workspace_forward_twice(name):
+    from paper_2606_29758_gb300 import _binding as B
+    cfg, D, up = _prepared(name)
+    N = up.N
+    for call in range(2):
+        out = {k: torch.full((N,), float("nan"), device="cuda") for k in OUTS}
+        loss = torch.full((1,), float("nan"), dtype=torch.float64, device="cuda")
+        B.ps_lmhead_ppo_fwd_noalloc(N, cfg.d, cfg.V, up.dcode, up.hid, D["W"], up.tok, up.oldlogp, up.adv, up.w,
+                                    cfg.eps, cfg.loss_scale, loss, out["lse"], out["logp"], out["ratio"],
+                                    out["coef"], out["row_loss"])
+        torch.cuda.synchronize()
+        rel = abs(loss.item() - up.loss.item()) / abs(up.loss.item())
+        assert rel < 1e-3, (call, rel)
+        for k in OUTS:
+            ref = getattr(up, k)[:N]
+            err = (out[k] - ref).abs().max().item()
+            assert err <= 2e-4 * max(1.0, ref.abs().max().item()), (call, k, err)
+
+
+def test_noalloc_rejects_problems_larger_than_its_scratch():
+    from paper_2606_29758_gb300 import _binding as B
+    with pytest.raises(B.PsppoError) as e:
+        B.ps_lmhead_ppo_fwd_noalloc(600_000, 3584, 152064, B.PS_DTYPE_BF16, None, None, None, None, None, None,
+                                    0.2, 1.0, None, None, None, None, None, None)
+    assert e.value.status == B.PS_ERR_UNSUPPORTED
