@@ -68,7 +68,8 @@ _SIGS = {
                                  _vp, _vp, _vp, _vp, _vp, _vp, _vp, _sz, _vp]),
     "ps_lmhead_ppo_bwd_workspace_size": (_sz, [_i64, _i32, _i32, _i32, _i64]),
     "ps_lmhead_ppo_bwd": (_i32, [_i64, _i32, _i32, _i32, _vp, _vp, _vp, _vp, _vp, _vp, _vp, _i32, _vp, _sz, _vp]),
-    "ps_diag_gemm_bf16": (_i32, [_i32, _i32, _i32, _i32, _i32, _vp, _i64, _vp, _i64, _vp, _i64, _i32, _vp, _sz, _vp]),
+    "ps_diag_gemm_bf16": (_i32, [_i32, _i32, _i32, _i32, _i32, _vp, _i64, _vp, _i64, _vp, _i64, _i32, _i32, _vp, _sz,
+                                 _vp]),
     "ps_diag_wait_timeout": (_i32, [_u64, _vp, _sz, _vp]),
     "ps_lmhead_ppo_fwd_noalloc": (_i32, [_i64, _i32, _i32, _i32, _vp, _vp, _vp, _vp, _vp, _vp, _f64, _f64,
                                          _vp, _vp, _vp, _vp, _vp, _vp, _vp]),
@@ -201,9 +202,10 @@ def ps_lmhead_ppo_bwd(N, d, V, dtype, Hpk, W, tok, lse, coef, dH, dW, flags, ws,
     _check(rc, "ps_lmhead_ppo_bwd")
 
 
-def ps_diag_gemm_bf16(M, N, K, a_mn_major, b_mn_major, A, lda, B, ldb, C, ldc, accumulate, ws, stream=None):
+def ps_diag_gemm_bf16(M, N, K, a_mn_major, b_mn_major, A, lda, B, ldb, C, ldc, accumulate, ws, cta_pair=1,
+                      stream=None):
     rc = lib().ps_diag_gemm_bf16(M, N, K, int(a_mn_major), int(b_mn_major), _ptr(A), lda, _ptr(B), ldb, _ptr(C), ldc,
-                                 int(accumulate), _ptr(ws), _nbytes(ws), _stream(stream))
+                                 int(accumulate), int(cta_pair), _ptr(ws), _nbytes(ws), _stream(stream))
     _check(rc, "ps_diag_gemm_bf16")
 
 

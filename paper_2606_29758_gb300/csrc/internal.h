@@ -28,9 +28,10 @@ int bwd_chunk_f32(int64_t rc, int d, int V, const float* Hpk, const float* W, co
                   const float* lse, const float* coef, float* dH, float* dW, int dw_accumulate, float* dz,
                   int64_t ldz, uint32_t* status, cudaStream_t s);
 
-// Plain tensor-core GEMM (test hook): C[M][N] (+)= sum_k A(m,k) B(k,n), f32 out.
+// Plain tensor-core GEMM (test hook): C[M][N] (+)= sum_k A(m,k) B(k,n), f32 out; pair selects
+// the CTA-pair kernel (256 x 256 tiles) instead of the single-CTA one (128 x 256).
 int gemm_bf16(int M, int N, int K, int a_mn, int b_mn, const void* A, int64_t lda, const void* B, int64_t ldb,
-              float* C, int64_t ldc, int accumulate, uint32_t* status, cudaStream_t s);
+              float* C, int64_t ldc, int accumulate, int pair, uint32_t* status, cudaStream_t s);
 
 // Bounded-wait self test: waits on an mbarrier nobody arrives at.
 int wait_timeout_probe(uint64_t timeout_ns, uint32_t* status, cudaStream_t s);

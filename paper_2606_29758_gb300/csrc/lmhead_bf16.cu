@@ -209,8 +209,9 @@ static bool map_mnmajor(CUtensorMap* m, const void* base, int64_t K, int64_t MN,
 }
 
 template <bool A_MN, bool B_MN, class Epi>
-static int launch_gemm(const CUtensorMap& ta, const CUtensorMap& tb, int64_t M, int64_t N, int64_t K, int splits,
-                       int band_m, const typename Epi::Params& ep, uint32_t* status, cudaStream_t s) {
+static int launch_gemm_single(const CUtensorMap& ta, const CUtensorMap& tb, int64_t M, int64_t N, int64_t K,
+                              int splits, int band_m, const typename Epi::Params& ep, uint32_t* status,
+                              cudaStream_t s) {
   Sched sc;
   sc.m_blocks = static_cast<int>((M + kBM - 1) / kBM);
   sc.n_blocks = static_cast<int>((N + kBN - 1) / kBN);
@@ -229,20 +230,70 @@ static int launch_gemm(const CUtensorMap& ta, const CUtensorMap& tb, int64_t M, 
   return cudaGetLastError() == cudaSuccess ? PS_OK : PS_ERR_CUDA;
 }
 
+// Number of CTA pairs of the pair kernel that fit on the device at once.
+template <class K>
+static int resident_pairs(K kern) {
+  cudaLaunchConfig_t cfg = {};
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeClusterDimension;
+  attr[0].val.clusterDim.x = 2;
+  attr[0].val.clusterDim.y = 1;
+  attr[0].val.clusterDim.z = 1;
+  cfg.gridDim = dim3(2 * (num_sms_current() / 2), 1, 1);
+  cfg.blockDim = dim3(kGemmThreads, 1, 1);
+  cfg.dynamicSmemBytes = kGemmPairSmemBytes;
+  cfg.attrs = attr;
+  cfg.numAttrs = 1;
+  int n = 0;
+  if (cudaOccupancyMaxActiveClusters(&n, reinterpret_cast<const void*>(kern), &cfg) != cudaSuccess || n <= 0) {
+    cudaGetLastError();
+    n = num_sms_current() / 2;
+  }
+  return n;
+}
+
+template <bool A_MN, bool B_MN, class Epi>
+static int launch_gemm_pair(const CUtensorMap& ta, const CUtensorMap& tb, int64_t M, int64_t N, int64_t K,
+                            int splits, int band_m, const typename Epi::Params& ep, uint32_t* status,
+                            cudaStream_t s) {
+  Sched sc;
+  sc.m_blocks = static_cast<int>((M + 255) / 256);
+  sc.n_blocks = static_cast<int>((N + kBN - 1) / kBN);
+  sc.splits = splits > 0 ? splits : sc.n_blocks;
+  sc.band_m = band_m > 0 ? band_m : 1;
+  sc.num_units = sc.m_blocks * sc.splits;
+  sc.num_kb = static_cast<int>((K + kBK - 1) / kBK);
+  if (sc.num_units == 0) return PS_OK;
+  if (sc.num_kb == 0) return PS_ERR_INVALID_ARG;
+  auto kern = umma_gemm_pair_kernel<A_MN, B_MN, Epi>;
+  if (cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                           static_cast<int>(kGemmPairSmemBytes)) != cudaSuccess)
+    return PS_ERR_CUDA;
+  const int pairs = sc.num_units < resident_pairs(kern) ? sc.num_units : resident_pairs(kern);
+  kern<<<2 * pairs, kGemmThreads, kGemmPairSmemBytes, s>>>(ta, tb, sc, ep, status, kDefaultTimeoutNs);
+  return cudaGetLastError() == cudaSuccess ? PS_OK : PS_ERR_CUDA;
+}
+
+// Row blocks of 128 rows per CTA (single) or 256 rows per CTA pair.
+template <bool A_MN, bool B_MN, class Epi>
+static int launch_gemm(bool pair, const CUtensorMap& ta, const CUtensorMap& tb, int64_t M, int64_t N, int64_t K,
+                       int splits, int band_m, const typename Epi::Params& ep, uint32_t* status, cudaStream_t s) {
+  return pair ? launch_gemm_pair<A_MN, B_MN, Epi>(ta, tb, M, N, K, splits, band_m, ep, status, s)
+              : launch_gemm_single<A_MN, B_MN, Epi>(ta, tb, M, N, K, splits, band_m, ep, status, s);
+}
+
 constexpr int kMaxFwdSplits = 16;
 int max_fwd_splits_bf16() { return kMaxFwdSplits; }
 
-// Pick the number of vocabulary ranges per 128-row block that minimises the number of
-// tile rounds of a static round-robin over `num_sms` CTAs (smaller on ties).
-int choose_fwd_splits_bf16(int64_t N, int V, int num_sms) {
-  const int64_t mb = (N + kBM - 1) / kBM;
-  const int64_t nb = (V + kBN - 1) / kBN;
+// Pick the number of vocabulary ranges per row block that minimises the number of tile
+// rounds of a static round-robin over `workers` (CTAs or CTA pairs); smaller on ties.
+static int choose_splits(int64_t m_blocks, int64_t n_blocks, int workers) {
   int best = 1;
   int64_t best_cost = INT64_MAX;
-  for (int s = 1; s <= kMaxFwdSplits && s <= nb; ++s) {
-    const int64_t units = mb * s;
-    const int64_t rounds = (units + num_sms - 1) / num_sms;
-    const int64_t cost = rounds * ((nb + s - 1) / s);
+  for (int s = 1; s <= kMaxFwdSplits && s <= n_blocks; ++s) {
+    const int64_t units = m_blocks * s;
+    const int64_t rounds = (units + workers - 1) / workers;
+    const int64_t cost = rounds * ((n_blocks + s - 1) / s);
     if (cost < best_cost) {
       best_cost = cost;
       best = s;
@@ -251,14 +302,33 @@ int choose_fwd_splits_bf16(int64_t N, int V, int num_sms) {
   return best;
 }
 
+// The product GEMMs run one CTA per 128 x 256 tile. The CTA-pair kernel (cta_group::2,
+// 256 x 256 per pair) does ~12% more work per clock, but on this part the pass is
+// power-capped, and at the cap the single-CTA kernel sustains the higher throughput
+// (343k vs 328k prefix tokens/s on the 7B-shaped step, same box, back to back): the pair
+// kernel draws more energy per FLOP, so the clock governor settles ~15% lower.
+constexpr bool kUsePairs = false;
+// Rows of a K-major B box: each CTA of a pair loads half of the 256-row B tile (16 KB per
+// stage, the size its ring slot holds and its expect-tx counts); a single CTA loads all of it.
+constexpr uint32_t kBRowsBox = kUsePairs ? 128 : kBN;
+
+int choose_fwd_splits_bf16(int64_t N, int V, int num_sms) {
+  const int64_t nb = (V + kBN - 1) / kBN;
+  if (kUsePairs) return choose_splits((N + 255) / 256, nb, num_sms / 2);
+  return choose_splits((N + kBM - 1) / kBM, nb, num_sms);
+}
+
 int fwd_gemm_bf16(int64_t N, int d, int V, const void* Hpk, const void* W, const int32_t* tok, float2* part,
                   float* ztok, int splits, uint32_t* status, cudaStream_t s) {
   CUtensorMap ta, tb;
-  if (!map_kmajor(&ta, Hpk, N, d, d, kBM) || !map_kmajor(&tb, W, V, d, d, kBN)) return PS_ERR_INVALID_ARG;
+  if (!map_kmajor(&ta, Hpk, N, d, d, kBM) || !map_kmajor(&tb, W, V, d, d, kBRowsBox)) return PS_ERR_INVALID_ARG;
   FwdLseEpi::Params ep{tok, static_cast<int>(N), V, part, ztok};
-  const int band = (num_sms_current() + splits - 1) / splits;
-  return launch_gemm<false, false, FwdLseEpi>(ta, tb, N, V, d, splits, band, ep, status, s);
+  const int workers = kUsePairs ? num_sms_current() / 2 : num_sms_current();
+  const int band = (workers + splits - 1) / splits;
+  return launch_gemm<false, false, FwdLseEpi>(kUsePairs, ta, tb, N, V, d, splits, band, ep, status, s);
 }
+
+constexpr int kBandBwd = 16;  // row blocks per band in the backward GEMMs
 
 int bwd_chunk_bf16(int64_t rc, int d, int V, const void* Hpk, const void* W, const int32_t* tok,
                    const float* lse, const float* coef, float* dH, float* dW, int dw_accumulate, void* dz,
@@ -266,39 +336,40 @@ int bwd_chunk_bf16(int64_t rc, int d, int V, const void* Hpk, const void* W, con
   int rcode;
   {
     CUtensorMap ta, tb;
-    if (!map_kmajor(&ta, Hpk, rc, d, d, kBM) || !map_kmajor(&tb, W, V, d, d, kBN)) return PS_ERR_INVALID_ARG;
+    if (!map_kmajor(&ta, Hpk, rc, d, d, kBM) || !map_kmajor(&tb, W, V, d, d, kBRowsBox)) return PS_ERR_INVALID_ARG;
     BwdDzEpi::Params ep{tok, lse, coef, static_cast<int>(rc), V, static_cast<__nv_bfloat16*>(dz), ldz};
-    rcode = launch_gemm<false, false, BwdDzEpi>(ta, tb, rc, V, d, 0, 16, ep, status, s);
+    rcode = launch_gemm<false, false, BwdDzEpi>(kUsePairs, ta, tb, rc, V, d, 0, kBandBwd, ep, status, s);
     if (rcode != PS_OK) return rcode;
   }
   if (dH) {
     CUtensorMap ta, tb;
     if (!map_kmajor(&ta, dz, rc, V, ldz, kBM) || !map_mnmajor(&tb, W, V, d, d)) return PS_ERR_INVALID_ARG;
     StoreF32Epi::Params ep{dH, d, static_cast<int>(rc), d, 0};
-    rcode = launch_gemm<false, true, StoreF32Epi>(ta, tb, rc, d, V, 0, 16, ep, status, s);
+    rcode = launch_gemm<false, true, StoreF32Epi>(kUsePairs, ta, tb, rc, d, V, 0, kBandBwd, ep, status, s);
     if (rcode != PS_OK) return rcode;
   }
   if (dW) {
     CUtensorMap ta, tb;
     if (!map_mnmajor(&ta, dz, rc, V, ldz) || !map_mnmajor(&tb, Hpk, rc, d, d)) return PS_ERR_INVALID_ARG;
     StoreF32Epi::Params ep{dW, d, V, d, dw_accumulate};
-    rcode = launch_gemm<true, true, StoreF32Epi>(ta, tb, V, d, rc, 0, 16, ep, status, s);
+    rcode = launch_gemm<true, true, StoreF32Epi>(kUsePairs, ta, tb, V, d, rc, 0, kBandBwd, ep, status, s);
     if (rcode != PS_OK) return rcode;
   }
   return PS_OK;
 }
 
 int gemm_bf16(int M, int N, int K, int a_mn, int b_mn, const void* A, int64_t lda, const void* B, int64_t ldb,
-              float* C, int64_t ldc, int accumulate, uint32_t* status, cudaStream_t s) {
+              float* C, int64_t ldc, int accumulate, int pair, uint32_t* status, cudaStream_t s) {
   CUtensorMap ta, tb;
+  const bool p = pair != 0;
   const bool oka = a_mn ? map_mnmajor(&ta, A, K, M, lda) : map_kmajor(&ta, A, M, K, lda, kBM);
-  const bool okb = b_mn ? map_mnmajor(&tb, B, K, N, ldb) : map_kmajor(&tb, B, N, K, ldb, kBN);
+  const bool okb = b_mn ? map_mnmajor(&tb, B, K, N, ldb) : map_kmajor(&tb, B, N, K, ldb, p ? 128 : kBN);
   if (!oka || !okb) return PS_ERR_INVALID_ARG;
   StoreF32Epi::Params ep{C, ldc, M, N, accumulate};
-  if (!a_mn && !b_mn) return launch_gemm<false, false, StoreF32Epi>(ta, tb, M, N, K, 0, 16, ep, status, s);
-  if (!a_mn && b_mn) return launch_gemm<false, true, StoreF32Epi>(ta, tb, M, N, K, 0, 16, ep, status, s);
-  if (a_mn && b_mn) return launch_gemm<true, true, StoreF32Epi>(ta, tb, M, N, K, 0, 16, ep, status, s);
-  return launch_gemm<true, false, StoreF32Epi>(ta, tb, M, N, K, 0, 16, ep, status, s);
+  if (!a_mn && !b_mn) return launch_gemm<false, false, StoreF32Epi>(p, ta, tb, M, N, K, 0, 16, ep, status, s);
+  if (!a_mn && b_mn) return launch_gemm<false, true, StoreF32Epi>(p, ta, tb, M, N, K, 0, 16, ep, status, s);
+  if (a_mn && b_mn) return launch_gemm<true, true, StoreF32Epi>(p, ta, tb, M, N, K, 0, 16, ep, status, s);
+  return launch_gemm<true, false, StoreF32Epi>(p, ta, tb, M, N, K, 0, 16, ep, status, s);
 }
 
 // ----------------------------------------------------------------------------- wait probe

@@ -600,15 +600,15 @@ int ps_lmhead_ppo_bwd(int64_t N, int d, int V, int dtype, const void* Hpk, const
 
 // ----------------------------------------------------------------------------- diagnostics
 int ps_diag_gemm_bf16(int M, int N, int K, int a_mn_major, int b_mn_major, const void* A, int64_t lda,
-                      const void* B, int64_t ldb, float* C, int64_t ldc, int accumulate, void* ws, size_t ws_bytes,
-                      ps_stream_t stream) {
+                      const void* B, int64_t ldb, float* C, int64_t ldc, int accumulate, int cta_pair, void* ws,
+                      size_t ws_bytes, ps_stream_t stream) {
   if (M < 1 || N < 1 || K < 1 || !A || !B || !C || ldc < N || ldc % 4 || !al16(C)) return PS_ERR_INVALID_ARG;
   if (lda < (a_mn_major ? M : K) || ldb < (b_mn_major ? N : K) || lda % 8 || ldb % 8) return PS_ERR_INVALID_ARG;
   if (!device_is_sm103()) return PS_ERR_UNSUPPORTED;
   cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
   int rc = begin_call(ws, ws_bytes, kWsHeader, s);
   if (rc != PS_OK) return rc;
-  return gemm_bf16(M, N, K, a_mn_major, b_mn_major, A, lda, B, ldb, C, ldc, accumulate, status_word(ws), s);
+  return gemm_bf16(M, N, K, a_mn_major, b_mn_major, A, lda, B, ldb, C, ldc, accumulate, cta_pair, status_word(ws), s);
 }
 
 int ps_diag_wait_timeout(uint64_t timeout_ns, void* ws, size_t ws_bytes, ps_stream_t stream) {

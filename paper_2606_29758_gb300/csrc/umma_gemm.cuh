@@ -241,4 +241,217 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
   }
 }
 
+
+// =============================================================================================
+// CTA-pair variant (tcgen05 cta_group::2). A cluster of two CTAs computes 256 x 256 output
+// tiles: each CTA loads its own 128 rows of A and one half (128 rows or columns) of B, so
+// a stage is 32 KB per CTA instead of 48 KB and six stages fit. The even CTA ("leader")
+// issues the MMAs for the pair (M = 256 split across the two CTAs' TMEM) and owns the
+// barriers that gate them:
+//   full[s]   (leader)  2 arrivals with expect-tx (one producer per CTA) + 64 KB of TMA bytes
+//   empty[s]  (both)    1 arrival: the leader's commit multicast to both CTAs
+//   tfull[a]  (both)    1 arrival: the leader's commit multicast to both CTAs
+//   tempty[a] (leader)  8 arrivals: one per epilogue warp of either CTA
+// Both CTAs walk the same sequence of units; every CTA reads its own TMEM lanes, i.e.
+// output rows 256 * m_pair + 128 * rank + lane.
+// =============================================================================================
+constexpr int kStagesPair = 6;
+constexpr uint32_t kHalfBBytes = 128 * kBK * 2;   // 16 KB: one CTA's half of the B tile
+
+struct GemmPairSmem {
+  uint8_t a[kStagesPair][kTileABytes];
+  uint8_t b[kStagesPair][kHalfBBytes];
+  uint64_t full[kStagesPair];
+  uint64_t empty[kStagesPair];
+  uint64_t tfull[2];
+  uint64_t tempty[2];
+  uint64_t drain;
+  uint32_t tmem_base;
+  int abort;
+};
+constexpr size_t kGemmPairSmemBytes = sizeof(GemmPairSmem) + 1024;
+
+template <bool A_MN, bool B_MN, class Epi>
+__global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kGemmThreads, 1)
+    umma_gemm_pair_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmB,
+                          const Sched sched, const typename Epi::Params ep, uint32_t* status,
+                          uint64_t timeout_ns) {
+  extern __shared__ uint8_t smem_raw[];
+  GemmPairSmem& sm =
+      *reinterpret_cast<GemmPairSmem*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
+  const int warp = threadIdx.x >> 5;
+  const int lane = threadIdx.x & 31;
+  const uint32_t rank = cluster_ctarank();
+  const bool leader = rank == 0;
+  const int pair = blockIdx.x >> 1;
+  const int npairs = gridDim.x >> 1;
+
+  if (threadIdx.x == 0) {
+    for (int s = 0; s < kStagesPair; ++s) {
+      mbar_init(&sm.full[s], 2);
+      mbar_init(&sm.empty[s], 1);
+    }
+    for (int a = 0; a < 2; ++a) {
+      mbar_init(&sm.tfull[a], 1);
+      mbar_init(&sm.tempty[a], 8);
+    }
+    mbar_init(&sm.drain, 1);
+    sm.abort = 0;
+    fence_mbar_init();
+  }
+  if (warp == 0 && lane == 0) {
+    tma_prefetch_desc(&tmA);
+    tma_prefetch_desc(&tmB);
+  }
+  if (warp == 1) {
+    tmem_alloc_pair(&sm.tmem_base, kTmemCols);
+    tmem_relinquish_pair();
+  }
+  tc_fence_before();
+  cluster_sync_all();  // barriers of both CTAs initialised before any remote arrival
+  tc_fence_after();
+  const uint32_t tmem_base = sm.tmem_base;
+  volatile int* abort = &sm.abort;
+
+  if (warp == 0) {
+    // ------------------------------------------------------------------ TMA producer (both CTAs)
+    if (lane == 0) {
+      uint32_t kc = 0;
+      bool ok = true;
+      for (int u = pair; ok && u < sched.num_units; u += npairs) {
+        int m_blk, split, n0, n1;
+        sched.unit(u, m_blk, split, n0, n1);
+        for (int nb = n0; ok && nb < n1; ++nb) {
+          for (int kb = 0; kb < sched.num_kb; ++kb, ++kc) {
+            const int s = kc % kStagesPair;
+            const uint32_t ph = (kc / kStagesPair) & 1u;
+            if (!mbar_wait(&sm.empty[s], ph ^ 1u, timeout_ns, abort)) { ok = false; break; }
+            const uint32_t lfull = mapa_shared(smem_addr(&sm.full[s]), 0);
+            mbar_arrive_expect_tx_cluster(lfull, kTileABytes + kHalfBBytes);
+            const int m0 = m_blk * 256 + static_cast<int>(rank) * 128;
+            const int nn0 = nb * kBN + static_cast<int>(rank) * 128;
+            const int k0 = kb * kBK;
+            if (A_MN) {
+              for (int i = 0; i < 2; ++i) tma_load_2d_pair(sm.a[s] + i * (kBK * 128), &tmA, lfull, m0 + i * 64, k0);
+            } else {
+              tma_load_2d_pair(sm.a[s], &tmA, lfull, k0, m0);
+            }
+            if (B_MN) {
+              for (int i = 0; i < 2; ++i) tma_load_2d_pair(sm.b[s] + i * (kBK * 128), &tmB, lfull, nn0 + i * 64, k0);
+            } else {
+              tma_load_2d_pair(sm.b[s], &tmB, lfull, k0, nn0);
+            }
+          }
+        }
+      }
+      if (!ok) {
+        *abort = 1;
+        raise_status(status, PS_DEV_TIMEOUT);
+        // the leader can see its stages land; the peer's barriers are remote, so it gives
+        // its own loads in flight a bounded grace period instead
+        if (leader) {
+          const uint32_t first = kc > kStagesPair ? kc - kStagesPair : 0;
+          for (uint32_t j = first; j < kc; ++j)
+            mbar_wait(&sm.full[j % kStagesPair], (j / kStagesPair) & 1u, timeout_ns, nullptr);
+        } else {
+          const uint64_t t0 = globaltimer_ns();
+          while (globaltimer_ns() - t0 < 2000000ull) {
+          }
+        }
+      }
+    }
+  } else if (warp == 1) {
+    // ------------------------------------------------------------------ MMA issuer (leader only)
+    if (lane == 0 && leader) {
+      constexpr uint32_t idesc = idesc_bf16_f32(256, kBN, A_MN, B_MN);
+      constexpr uint32_t a_lbo = A_MN ? kBK * 128 : 16, a_step = A_MN ? 2048 : 32;
+      constexpr uint32_t b_lbo = B_MN ? kBK * 128 : 16, b_step = B_MN ? 2048 : 32;
+      uint32_t kc = 0, tile = 0;
+      bool ok = true;
+      for (int u = pair; ok && u < sched.num_units; u += npairs) {
+        int m_blk, split, n0, n1;
+        sched.unit(u, m_blk, split, n0, n1);
+        for (int nb = n0; ok && nb < n1; ++nb, ++tile) {
+          const uint32_t acc = tile & 1u;
+          const uint32_t aph = (tile >> 1) & 1u;
+          if (!mbar_wait(&sm.tempty[acc], aph ^ 1u, timeout_ns, abort)) { ok = false; break; }
+          tc_fence_after();
+          const uint32_t d_tmem = tmem_base + acc * kBN;
+          for (int kb = 0; kb < sched.num_kb; ++kb, ++kc) {
+            const int s = kc % kStagesPair;
+            const uint32_t ph = (kc / kStagesPair) & 1u;
+            if (!mbar_wait(&sm.full[s], ph, timeout_ns, abort)) { ok = false; break; }
+            tc_fence_after();
+            const uint32_t a_base = smem_addr(sm.a[s]);
+            const uint32_t b_base = smem_addr(sm.b[s]);
+#pragma unroll
+            for (int k = 0; k < kBK / 16; ++k) {
+              const uint64_t ad = smem_desc_sw128(a_base + k * a_step, a_lbo, 1024);
+              const uint64_t bd = smem_desc_sw128(b_base + k * b_step, b_lbo, 1024);
+              umma_bf16_pair(d_tmem, ad, bd, idesc, (kb | k) != 0 ? 1u : 0u);
+            }
+            umma_commit_pair_multicast(&sm.empty[s], 0x3);
+          }
+          if (ok) umma_commit_pair_multicast(&sm.tfull[acc], 0x3);
+        }
+      }
+      if (!ok) {
+        *abort = 1;
+        raise_status(status, PS_DEV_TIMEOUT);
+        umma_commit_pair_multicast(&sm.drain, 0x1);
+        mbar_wait(&sm.drain, 0, timeout_ns, nullptr);
+      }
+    }
+  } else {
+    // ------------------------------------------------------------------ epilogue (both CTAs)
+    const int quad = warp & 3;
+    const int row_in_tile = quad * 32 + lane;
+    const uint32_t ltempty0 = mapa_shared(smem_addr(&sm.tempty[0]), 0);
+    const uint32_t ltempty1 = mapa_shared(smem_addr(&sm.tempty[1]), 0);
+    typename Epi::State st;
+    uint32_t tile = 0;
+    bool ok = true;
+    for (int u = pair; ok && u < sched.num_units; u += npairs) {
+      int m_blk, split, n0, n1;
+      sched.unit(u, m_blk, split, n0, n1);
+      const int row = m_blk * 256 + static_cast<int>(rank) * 128 + row_in_tile;
+      Epi::begin_unit(ep, st, row, split);
+      for (int nb = n0; nb < n1; ++nb, ++tile) {
+        const uint32_t acc = tile & 1u;
+        const uint32_t aph = (tile >> 1) & 1u;
+        int got = 0;
+        if (lane == 0) got = mbar_wait(&sm.tfull[acc], aph, timeout_ns, abort) ? 1 : 0;
+        got = __shfl_sync(0xffffffffu, got, 0);
+        if (!got) { ok = false; break; }
+        tc_fence_after();
+        const uint32_t t_row = tmem_base + (static_cast<uint32_t>(quad * 32) << 16) + acc * kBN;
+#pragma unroll 1
+        for (int c = 0; c < kBN / 32; ++c) {
+          uint32_t r[32];
+          tmem_ld32(t_row + c * 32, r);
+          tmem_ld_wait();
+          if (c == kBN / 32 - 1) {
+            tc_fence_before();
+            __syncwarp();
+            if (lane == 0) mbar_arrive_cluster(acc ? ltempty1 : ltempty0);
+          }
+          Epi::chunk(ep, st, row, nb * kBN + c * 32, r);
+        }
+      }
+      if (ok) Epi::end_unit(ep, st, row, split);
+    }
+    if (!ok) {
+      *abort = 1;
+      raise_status(status, PS_DEV_TIMEOUT);
+    }
+  }
+
+  tc_fence_before();
+  cluster_sync_all();  // no remote arrival or multicast commit can target an exited CTA
+  if (warp == 1) {
+    tc_fence_after();
+    tmem_dealloc_pair(tmem_base, kTmemCols);
+  }
+}
+
 }  // namespace psk
