@@ -20,13 +20,14 @@ extern "C" {
  * A(m, k) is A[m*lda + k] (a_mn_major = 0, K-major) or A[k*lda + m] (a_mn_major = 1);
  * B(k, n) is B[n*ldb + k] (b_mn_major = 0, K-major) or B[k*ldb + n] (b_mn_major = 1).
  * C is f32 [M][ldc], overwritten (accumulate = 0) or added to (accumulate = 1).
- * cta_pair = 1 runs the kernel the library uses: two CTAs of a cluster share each
- * 256 x 256 tile (tcgen05 cta_group::2); cta_pair = 0 runs one CTA per 128 x 256 tile.
+ * variant selects the kernel: 0 = one CTA per 128 x 256 tile (the forward and the logit
+ * recompute), 1 = two CTAs of a cluster per 256 x 256 tile (tcgen05 cta_group::2), 2 = one
+ * CTA per 256 x 256 tile as two M = 128 halves sharing B (dH and dW).
  * lda, ldb multiples of 8; ldc a multiple of 4; 16-byte aligned A, B, C.
  * ws: at least 256 bytes. sm_103 only (PS_ERR_UNSUPPORTED elsewhere).
  */
 int ps_diag_gemm_bf16(int M, int N, int K, int a_mn_major, int b_mn_major, const void* A, int64_t lda,
-                      const void* B, int64_t ldb, float* C, int64_t ldc, int accumulate, int cta_pair,
+                      const void* B, int64_t ldb, float* C, int64_t ldc, int accumulate, int variant,
                       void* ws, size_t ws_bytes, ps_stream_t stream);
 
 /*

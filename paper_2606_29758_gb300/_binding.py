@@ -202,10 +202,10 @@ def ps_lmhead_ppo_bwd(N, d, V, dtype, Hpk, W, tok, lse, coef, dH, dW, flags, ws,
     _check(rc, "ps_lmhead_ppo_bwd")
 
 
-def ps_diag_gemm_bf16(M, N, K, a_mn_major, b_mn_major, A, lda, B, ldb, C, ldc, accumulate, ws, cta_pair=1,
+def ps_diag_gemm_bf16(M, N, K, a_mn_major, b_mn_major, A, lda, B, ldb, C, ldc, accumulate, ws, variant=0,
                       stream=None):
     rc = lib().ps_diag_gemm_bf16(M, N, K, int(a_mn_major), int(b_mn_major), _ptr(A), lda, _ptr(B), ldb, _ptr(C), ldc,
-                                 int(accumulate), int(cta_pair), _ptr(ws), _nbytes(ws), _stream(stream))
+                                 int(accumulate), int(variant), _ptr(ws), _nbytes(ws), _stream(stream))
     _check(rc, "ps_diag_gemm_bf16")
 
 

@@ -12,7 +12,7 @@ int device_is_sm103();
 // Forward GEMM with the online-logsumexp epilogue. part: [splits][N] (max2, sum) pairs
 // (max in log2 units); ztok: [N] chosen-token logit.
 int max_fwd_splits_bf16();
-int choose_fwd_splits_bf16(int64_t N, int V, int num_sms);
+int choose_fwd_splits_bf16(int64_t N, int d, int V, int num_sms);
 int fwd_gemm_bf16(int64_t N, int d, int V, const void* Hpk, const void* W, const int32_t* tok, float2* part,
                   float* ztok, int splits, uint32_t* status, cudaStream_t s);
 int fwd_splits_f32(int V);
@@ -28,10 +28,10 @@ int bwd_chunk_f32(int64_t rc, int d, int V, const float* Hpk, const float* W, co
                   const float* lse, const float* coef, float* dH, float* dW, int dw_accumulate, float* dz,
                   int64_t ldz, uint32_t* status, cudaStream_t s);
 
-// Plain tensor-core GEMM (test hook): C[M][N] (+)= sum_k A(m,k) B(k,n), f32 out; pair selects
-// the CTA-pair kernel (256 x 256 tiles) instead of the single-CTA one (128 x 256).
+// Plain tensor-core GEMM (test hook): C[M][N] (+)= sum_k A(m,k) B(k,n), f32 out. variant: 0 one
+// CTA per 128 x 256 tile, 1 a CTA pair per 256 x 256 tile, 2 one CTA per 256 x 256 tile.
 int gemm_bf16(int M, int N, int K, int a_mn, int b_mn, const void* A, int64_t lda, const void* B, int64_t ldb,
-              float* C, int64_t ldc, int accumulate, int pair, uint32_t* status, cudaStream_t s);
+              float* C, int64_t ldc, int accumulate, int variant, uint32_t* status, cudaStream_t s);
 
 // Bounded-wait self test: waits on an mbarrier nobody arrives at.
 int wait_timeout_probe(uint64_t timeout_ns, uint32_t* status, cudaStream_t s);

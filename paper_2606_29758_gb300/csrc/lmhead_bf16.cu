@@ -208,12 +208,12 @@ static bool map_mnmajor(CUtensorMap* m, const void* base, int64_t K, int64_t MN,
   return make_map(m, base, MN, K, pitch_elems * 2, 64, kBK);
 }
 
-template <bool A_MN, bool B_MN, class Epi>
+template <bool A_MN, bool B_MN, class Epi, int HALVES = 1>
 static int launch_gemm_single(const CUtensorMap& ta, const CUtensorMap& tb, int64_t M, int64_t N, int64_t K,
                               int splits, int band_m, const typename Epi::Params& ep, uint32_t* status,
                               cudaStream_t s) {
   Sched sc;
-  sc.m_blocks = static_cast<int>((M + kBM - 1) / kBM);
+  sc.m_blocks = static_cast<int>((M + kBM * HALVES - 1) / (kBM * HALVES));
   sc.n_blocks = static_cast<int>((N + kBN - 1) / kBN);
   sc.splits = splits > 0 ? splits : sc.n_blocks;
   sc.band_m = band_m > 0 ? band_m : 1;
@@ -221,12 +221,13 @@ static int launch_gemm_single(const CUtensorMap& ta, const CUtensorMap& tb, int6
   sc.num_kb = static_cast<int>((K + kBK - 1) / kBK);
   if (sc.num_units == 0) return PS_OK;
   if (sc.num_kb == 0) return PS_ERR_INVALID_ARG;
-  auto kern = umma_gemm_kernel<A_MN, B_MN, Epi>;
-  if (cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, static_cast<int>(kGemmSmemBytes)) !=
+  auto kern = umma_gemm_kernel<A_MN, B_MN, Epi, HALVES>;
+  constexpr size_t smem = gemm_smem_bytes<HALVES>();
+  if (cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, static_cast<int>(smem)) !=
       cudaSuccess)
     return PS_ERR_CUDA;
   const int grid = sc.num_units < num_sms_current() ? sc.num_units : num_sms_current();
-  kern<<<grid, kGemmThreads, kGemmSmemBytes, s>>>(ta, tb, sc, ep, status, kDefaultTimeoutNs);
+  kern<<<grid, kGemmThreads, smem, s>>>(ta, tb, sc, ep, status, kDefaultTimeoutNs);
   return cudaGetLastError() == cudaSuccess ? PS_OK : PS_ERR_CUDA;
 }
 
@@ -285,50 +286,79 @@ static int launch_gemm(bool pair, const CUtensorMap& ta, const CUtensorMap& tb, 
 constexpr int kMaxFwdSplits = 16;
 int max_fwd_splits_bf16() { return kMaxFwdSplits; }
 
-// Pick the number of vocabulary ranges per row block that minimises the number of tile
-// rounds of a static round-robin over `workers` (CTAs or CTA pairs); smaller on ties.
-static int choose_splits(int64_t m_blocks, int64_t n_blocks, int workers) {
-  int best = 1;
-  int64_t best_cost = INT64_MAX;
-  for (int s = 1; s <= kMaxFwdSplits && s <= n_blocks; ++s) {
+// Pick the number of vocabulary ranges per row block: the makespan of a static round-robin
+// over `workers` (CTAs or CTA pairs), in tiles, is rounds x tiles per unit. Among the split
+// counts within 1% of the best makespan, take the smallest: fewer ranges mean wider bands of
+// row blocks and fewer passes over W.
+static int choose_splits(int64_t m_blocks, int64_t n_blocks, int workers, int min_splits = 1) {
+  auto cost = [&](int s) {
     const int64_t units = m_blocks * s;
-    const int64_t rounds = (units + workers - 1) / workers;
-    const int64_t cost = rounds * ((n_blocks + s - 1) / s);
-    if (cost < best_cost) {
-      best_cost = cost;
-      best = s;
-    }
-  }
-  return best;
+    return ((units + workers - 1) / workers) * ((n_blocks + s - 1) / s);
+  };
+  const int hi = static_cast<int>(n_blocks < kMaxFwdSplits ? n_blocks : kMaxFwdSplits);
+  if (min_splits > hi) return hi;
+  int64_t best = INT64_MAX;
+  for (int s = min_splits; s <= hi; ++s) best = cost(s) < best ? cost(s) : best;
+  for (int s = min_splits; s <= hi; ++s)
+    if (cost(s) * 100 <= best * 101) return s;
+  return min_splits;
 }
 
-// The product GEMMs run one CTA per 128 x 256 tile. The CTA-pair kernel (cta_group::2,
-// 256 x 256 per pair) does ~12% more work per clock, but on this part the pass is
-// power-capped, and at the cap the single-CTA kernel sustains the higher throughput
-// (343k vs 328k prefix tokens/s on the 7B-shaped step, same box, back to back): the pair
-// kernel draws more energy per FLOP, so the clock governor settles ~15% lower.
 constexpr bool kUsePairs = false;
 // Rows of a K-major B box: each CTA of a pair loads half of the 256-row B tile (16 KB per
 // stage, the size its ring slot holds and its expect-tx counts); a single CTA loads all of it.
 constexpr uint32_t kBRowsBox = kUsePairs ? 128 : kBN;
+// Tile height of the forward and of the logit recompute in 128-row halves (see GemmCfg). The
+// forward gains from the wide tile (fewer operand bytes per FLOP) even though its epilogue is
+// then not overlapped; the recompute, whose epilogue also writes dZ, does better with
+// 128-row tiles and double-buffered accumulators (7B-shaped step, measured back to back).
+constexpr int kFwdHalves = 2;
+constexpr int kRecHalves = 1;
 
-int choose_fwd_splits_bf16(int64_t N, int V, int num_sms) {
+// The forward keeps one band of row blocks in flight; every CTA of the band sweeps its
+// vocabulary range and re-reads its row block for every vocabulary tile, so the band's
+// hidden rows must stay in L2 (129 MB) next to the W tiles being streamed. Cap them at a
+// third of L2; that sets the minimum number of vocabulary ranges per row block.
+constexpr double kFwdBandL2Bytes = 43e6;
+
+static int fwd_min_splits(int d, int workers);
+
+int choose_fwd_splits_bf16(int64_t N, int d, int V, int num_sms) {
   const int64_t nb = (V + kBN - 1) / kBN;
-  if (kUsePairs) return choose_splits((N + 255) / 256, nb, num_sms / 2);
-  return choose_splits((N + kBM - 1) / kBM, nb, num_sms);
+  const int rows = kUsePairs ? 256 : kBM * kFwdHalves;
+  const int workers = kUsePairs ? num_sms / 2 : num_sms;
+  int lo = fwd_min_splits(d, workers);
+  if (lo > nb) lo = static_cast<int>(nb);
+  if (lo > kMaxFwdSplits) lo = kMaxFwdSplits;
+  return choose_splits((N + rows - 1) / rows, nb, workers, lo);
+}
+
+static int fwd_min_splits(int d, int workers) {
+  const int rows = kUsePairs ? 256 : kBM * kFwdHalves;
+  const double block_bytes = static_cast<double>(rows) * d * 2.0;
+  int band_max = static_cast<int>(kFwdBandL2Bytes / block_bytes);
+  if (band_max < 1) band_max = 1;
+  return (workers + band_max - 1) / band_max;
 }
 
 int fwd_gemm_bf16(int64_t N, int d, int V, const void* Hpk, const void* W, const int32_t* tok, float2* part,
                   float* ztok, int splits, uint32_t* status, cudaStream_t s) {
   CUtensorMap ta, tb;
-  if (!map_kmajor(&ta, Hpk, N, d, d, kBM) || !map_kmajor(&tb, W, V, d, d, kBRowsBox)) return PS_ERR_INVALID_ARG;
+  static_assert(!kUsePairs, "the wide forward tile is a single-CTA kernel");
+  if (!map_kmajor(&ta, Hpk, N, d, d, kBM * kFwdHalves) || !map_kmajor(&tb, W, V, d, d, kBRowsBox))
+    return PS_ERR_INVALID_ARG;
   FwdLseEpi::Params ep{tok, static_cast<int>(N), V, part, ztok};
-  const int workers = kUsePairs ? num_sms_current() / 2 : num_sms_current();
+  const int workers = num_sms_current();
   const int band = (workers + splits - 1) / splits;
-  return launch_gemm<false, false, FwdLseEpi>(kUsePairs, ta, tb, N, V, d, splits, band, ep, status, s);
+  return launch_gemm_single<false, false, FwdLseEpi, kFwdHalves>(ta, tb, N, V, d, splits, band, ep, status, s);
 }
 
-constexpr int kBandBwd = 16;  // row blocks per band in the backward GEMMs
+// Bands (row blocks walked together) of the backward GEMMs. Recompute: 48 row blocks share
+// each W tile (their hidden rows, 44 MB at d = 3584, stay in L2). dH and dW: one row block
+// per band, i.e. all column tiles of a row block run side by side, so each panel of dZ (the
+// large operand) is read from DRAM once and the small operand once per wave.
+constexpr int kBandRecompute = 48;
+constexpr int kBandGrad = 1;
 
 int bwd_chunk_bf16(int64_t rc, int d, int V, const void* Hpk, const void* W, const int32_t* tok,
                    const float* lse, const float* coef, float* dH, float* dW, int dw_accumulate, void* dz,
@@ -336,40 +366,54 @@ int bwd_chunk_bf16(int64_t rc, int d, int V, const void* Hpk, const void* W, con
   int rcode;
   {
     CUtensorMap ta, tb;
-    if (!map_kmajor(&ta, Hpk, rc, d, d, kBM) || !map_kmajor(&tb, W, V, d, d, kBRowsBox)) return PS_ERR_INVALID_ARG;
+    if (!map_kmajor(&ta, Hpk, rc, d, d, kBM * kRecHalves) || !map_kmajor(&tb, W, V, d, d, kBRowsBox))
+      return PS_ERR_INVALID_ARG;
     BwdDzEpi::Params ep{tok, lse, coef, static_cast<int>(rc), V, static_cast<__nv_bfloat16*>(dz), ldz};
-    rcode = launch_gemm<false, false, BwdDzEpi>(kUsePairs, ta, tb, rc, V, d, 0, kBandBwd, ep, status, s);
+    rcode = launch_gemm_single<false, false, BwdDzEpi, kRecHalves>(ta, tb, rc, V, d, 0, kBandRecompute / kRecHalves,
+                                                                    ep, status, s);
     if (rcode != PS_OK) return rcode;
   }
+  // dH (K = V) and dW (K = chunk rows) have long K loops: one CTA computes a 256 x 256 tile
+  // as two M = 128 halves that share each B stage (a third fewer operand bytes per FLOP).
   if (dH) {
     CUtensorMap ta, tb;
-    if (!map_kmajor(&ta, dz, rc, V, ldz, kBM) || !map_mnmajor(&tb, W, V, d, d)) return PS_ERR_INVALID_ARG;
+    if (!map_kmajor(&ta, dz, rc, V, ldz, 2 * kBM) || !map_mnmajor(&tb, W, V, d, d)) return PS_ERR_INVALID_ARG;
     StoreF32Epi::Params ep{dH, d, static_cast<int>(rc), d, 0};
-    rcode = launch_gemm<false, true, StoreF32Epi>(kUsePairs, ta, tb, rc, d, V, 0, kBandBwd, ep, status, s);
+    rcode = launch_gemm_single<false, true, StoreF32Epi, 2>(ta, tb, rc, d, V, 0, kBandGrad, ep, status, s);
     if (rcode != PS_OK) return rcode;
   }
   if (dW) {
     CUtensorMap ta, tb;
     if (!map_mnmajor(&ta, dz, rc, V, ldz) || !map_mnmajor(&tb, Hpk, rc, d, d)) return PS_ERR_INVALID_ARG;
     StoreF32Epi::Params ep{dW, d, V, d, dw_accumulate};
-    rcode = launch_gemm<true, true, StoreF32Epi>(kUsePairs, ta, tb, V, d, rc, 0, kBandBwd, ep, status, s);
+    rcode = launch_gemm_single<true, true, StoreF32Epi, 2>(ta, tb, V, d, rc, 0, kBandGrad, ep, status, s);
     if (rcode != PS_OK) return rcode;
   }
   return PS_OK;
 }
 
 int gemm_bf16(int M, int N, int K, int a_mn, int b_mn, const void* A, int64_t lda, const void* B, int64_t ldb,
-              float* C, int64_t ldc, int accumulate, int pair, uint32_t* status, cudaStream_t s) {
+              float* C, int64_t ldc, int accumulate, int variant, uint32_t* status, cudaStream_t s) {
+  if (variant < 0 || variant > 2) return PS_ERR_INVALID_ARG;
   CUtensorMap ta, tb;
-  const bool p = pair != 0;
-  const bool oka = a_mn ? map_mnmajor(&ta, A, K, M, lda) : map_kmajor(&ta, A, M, K, lda, kBM);
-  const bool okb = b_mn ? map_mnmajor(&tb, B, K, N, ldb) : map_kmajor(&tb, B, N, K, ldb, p ? 128 : kBN);
+  const uint32_t a_rows = variant == 2 ? 2 * kBM : kBM;     // K-major A box rows
+  const uint32_t b_rows = variant == 1 ? 128 : kBN;         // K-major B box rows (half per CTA of a pair)
+  const bool oka = a_mn ? map_mnmajor(&ta, A, K, M, lda) : map_kmajor(&ta, A, M, K, lda, a_rows);
+  const bool okb = b_mn ? map_mnmajor(&tb, B, K, N, ldb) : map_kmajor(&tb, B, N, K, ldb, b_rows);
   if (!oka || !okb) return PS_ERR_INVALID_ARG;
   StoreF32Epi::Params ep{C, ldc, M, N, accumulate};
-  if (!a_mn && !b_mn) return launch_gemm<false, false, StoreF32Epi>(p, ta, tb, M, N, K, 0, 16, ep, status, s);
-  if (!a_mn && b_mn) return launch_gemm<false, true, StoreF32Epi>(p, ta, tb, M, N, K, 0, 16, ep, status, s);
-  if (a_mn && b_mn) return launch_gemm<true, true, StoreF32Epi>(p, ta, tb, M, N, K, 0, 16, ep, status, s);
-  return launch_gemm<true, false, StoreF32Epi>(p, ta, tb, M, N, K, 0, 16, ep, status, s);
+  using E = StoreF32Epi;
+  if (variant == 2) {
+    if (!a_mn && !b_mn) return launch_gemm_single<false, false, E, 2>(ta, tb, M, N, K, 0, 16, ep, status, s);
+    if (!a_mn && b_mn) return launch_gemm_single<false, true, E, 2>(ta, tb, M, N, K, 0, 16, ep, status, s);
+    if (a_mn && b_mn) return launch_gemm_single<true, true, E, 2>(ta, tb, M, N, K, 0, 16, ep, status, s);
+    return launch_gemm_single<true, false, E, 2>(ta, tb, M, N, K, 0, 16, ep, status, s);
+  }
+  const bool p = variant == 1;
+  if (!a_mn && !b_mn) return launch_gemm<false, false, E>(p, ta, tb, M, N, K, 0, 16, ep, status, s);
+  if (!a_mn && b_mn) return launch_gemm<false, true, E>(p, ta, tb, M, N, K, 0, 16, ep, status, s);
+  if (a_mn && b_mn) return launch_gemm<true, true, E>(p, ta, tb, M, N, K, 0, 16, ep, status, s);
+  return launch_gemm<true, false, E>(p, ta, tb, M, N, K, 0, 16, ep, status, s);
 }
 
 // ----------------------------------------------------------------------------- wait probe

@@ -531,7 +531,7 @@ int ps_lmhead_ppo_fwd(int64_t N, int d, int V, int dtype, const void* Hpk, const
   if (N == 0) return cudaMemsetAsync(loss, 0, sizeof(double), s) == cudaSuccess ? PS_OK : PS_ERR_CUDA;
   int splits;
   if (dtype == PS_DTYPE_BF16) {
-    splits = choose_fwd_splits_bf16(N, V, num_sms_current());
+    splits = choose_fwd_splits_bf16(N, d, V, num_sms_current());
     rc = fwd_gemm_bf16(N, d, V, Hpk, W, tok, f.part, f.ztok, splits, status_word(ws), s);
   } else {
     splits = fwd_splits_f32(V);
@@ -600,7 +600,7 @@ int ps_lmhead_ppo_bwd(int64_t N, int d, int V, int dtype, const void* Hpk, const
 
 // ----------------------------------------------------------------------------- diagnostics
 int ps_diag_gemm_bf16(int M, int N, int K, int a_mn_major, int b_mn_major, const void* A, int64_t lda,
-                      const void* B, int64_t ldb, float* C, int64_t ldc, int accumulate, int cta_pair, void* ws,
+                      const void* B, int64_t ldb, float* C, int64_t ldc, int accumulate, int variant, void* ws,
                       size_t ws_bytes, ps_stream_t stream) {
   if (M < 1 || N < 1 || K < 1 || !A || !B || !C || ldc < N || ldc % 4 || !al16(C)) return PS_ERR_INVALID_ARG;
   if (lda < (a_mn_major ? M : K) || ldb < (b_mn_major ? N : K) || lda % 8 || ldb % 8) return PS_ERR_INVALID_ARG;
@@ -608,7 +608,7 @@ int ps_diag_gemm_bf16(int M, int N, int K, int a_mn_major, int b_mn_major, const
   cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
   int rc = begin_call(ws, ws_bytes, kWsHeader, s);
   if (rc != PS_OK) return rc;
-  return gemm_bf16(M, N, K, a_mn_major, b_mn_major, A, lda, B, ldb, C, ldc, accumulate, cta_pair, status_word(ws), s);
+  return gemm_bf16(M, N, K, a_mn_major, b_mn_major, A, lda, B, ldb, C, ldc, accumulate, variant, status_word(ws), s);
 }
 
 int ps_diag_wait_timeout(uint64_t timeout_ns, void* ws, size_t ws_bytes, ps_stream_t stream) {

@@ -55,31 +55,51 @@ struct Sched {
   }
 };
 
-struct GemmSmem {
+// HALVES = 1: 128 x 256 tiles, two TMEM accumulators (double-buffered), 4-stage 48 KB ring.
+// HALVES = 2: 256 x 256 tiles computed as two M = 128 MMAs that share each B stage, one
+// accumulator pair filling TMEM (not double-buffered), 3-stage 64 KB ring. The wide tile reads
+// a third fewer operand bytes per FLOP; the epilogue of a tile is not overlapped with the next
+// tile's main loop. Each epilogue thread owns one row of each half (two epilogue states).
+template <int HALVES>
+struct GemmCfg {
+  static constexpr int kStagesH = HALVES == 1 ? 4 : 3;
+  static constexpr int kRows = kBM * HALVES;                  // rows per tile
+  static constexpr uint32_t kABytes = kTileABytes * HALVES;   // A bytes per stage
+  static constexpr int kAccBufs = HALVES == 1 ? 2 : 1;        // accumulator buffers in TMEM
+};
+
+template <int HALVES>
+struct GemmSmemT {
   // 1024-byte aligned tile ring first (128-byte swizzle atoms repeat every 1 KB)
-  uint8_t a[kStages][kTileABytes];
-  uint8_t b[kStages][kTileBBytes];
-  uint64_t full[kStages];
-  uint64_t empty[kStages];
+  uint8_t a[GemmCfg<HALVES>::kStagesH][GemmCfg<HALVES>::kABytes];
+  uint8_t b[GemmCfg<HALVES>::kStagesH][kTileBBytes];
+  uint64_t full[GemmCfg<HALVES>::kStagesH];
+  uint64_t empty[GemmCfg<HALVES>::kStagesH];
   uint64_t tfull[2];
   uint64_t tempty[2];
   uint64_t drain;
   uint32_t tmem_base;
   int abort;
 };
-constexpr size_t kGemmSmemBytes = sizeof(GemmSmem) + 1024;  // + alignment slack
+template <int HALVES>
+constexpr size_t gemm_smem_bytes() { return sizeof(GemmSmemT<HALVES>) + 1024; }  // + alignment slack
+constexpr size_t kGemmSmemBytes = gemm_smem_bytes<1>();
 
-template <bool A_MN, bool B_MN, class Epi>
+template <bool A_MN, bool B_MN, class Epi, int HALVES = 1>
 __global__ void __launch_bounds__(kGemmThreads, 1)
     umma_gemm_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmB,
                      const Sched sched, const typename Epi::Params ep, uint32_t* status, uint64_t timeout_ns) {
+  using Cfg = GemmCfg<HALVES>;
+  constexpr int S = Cfg::kStagesH;
+  constexpr int NB = Cfg::kAccBufs;
   extern __shared__ uint8_t smem_raw[];
-  GemmSmem& sm = *reinterpret_cast<GemmSmem*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
+  GemmSmemT<HALVES>& sm =
+      *reinterpret_cast<GemmSmemT<HALVES>*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
   const int warp = threadIdx.x >> 5;
   const int lane = threadIdx.x & 31;
 
   if (threadIdx.x == 0) {
-    for (int s = 0; s < kStages; ++s) {
+    for (int s = 0; s < S; ++s) {
       mbar_init(&sm.full[s], 1);
       mbar_init(&sm.empty[s], 1);
     }
@@ -115,16 +135,16 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
         sched.unit(u, m_blk, split, n0, n1);
         for (int nb = n0; ok && nb < n1; ++nb) {
           for (int kb = 0; kb < sched.num_kb; ++kb, ++kc) {
-            const int s = kc % kStages;
-            const uint32_t ph = (kc / kStages) & 1u;
+            const int s = kc % S;
+            const uint32_t ph = (kc / S) & 1u;
             if (!mbar_wait(&sm.empty[s], ph ^ 1u, timeout_ns, abort)) { ok = false; break; }
-            mbar_arrive_expect_tx(&sm.full[s], kTileABytes + kTileBBytes);
-            const int m0 = m_blk * kBM, nn0 = nb * kBN, k0 = kb * kBK;
+            mbar_arrive_expect_tx(&sm.full[s], Cfg::kABytes + kTileBBytes);
+            const int m0 = m_blk * Cfg::kRows, nn0 = nb * kBN, k0 = kb * kBK;
             if (A_MN) {
-              for (int i = 0; i < kBM / 64; ++i)
+              for (int i = 0; i < Cfg::kRows / 64; ++i)
                 tma_load_2d(sm.a[s] + i * (kBK * 128), &tmA, &sm.full[s], m0 + i * 64, k0);
             } else {
-              tma_load_2d(sm.a[s], &tmA, &sm.full[s], k0, m0);
+              tma_load_2d(sm.a[s], &tmA, &sm.full[s], k0, m0);   // box of kRows rows
             }
             if (B_MN) {
               for (int i = 0; i < kBN / 64; ++i)
@@ -139,9 +159,8 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
         *abort = 1;
         raise_status(status, PS_DEV_TIMEOUT);
         // let the loads already issued land before the CTA can exit
-        const uint32_t first = kc > kStages ? kc - kStages : 0;
-        for (uint32_t j = first; j < kc; ++j)
-          mbar_wait(&sm.full[j % kStages], (j / kStages) & 1u, timeout_ns, nullptr);
+        const uint32_t first = kc > static_cast<uint32_t>(S) ? kc - S : 0;
+        for (uint32_t j = first; j < kc; ++j) mbar_wait(&sm.full[j % S], (j / S) & 1u, timeout_ns, nullptr);
       }
     }
   } else if (warp == 1) {
@@ -151,6 +170,8 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
       // K-major: 8-row groups 1024 B apart; a 16-deep K step is 32 B inside the swizzle atom.
       // MN-major: 64-element atoms kBK*128 B apart (LBO); 8-row K groups 1024 B apart (SBO);
       //           a 16-deep K step is 16 rows = 2048 B.
+      // The second half of a wide tile (rows 128..255) starts 16 KB into the A stage in both
+      // layouts (128 K-major rows of 128 B, or two MN-major atoms of 8 KB).
       constexpr uint32_t a_lbo = A_MN ? kBK * 128 : 16, a_step = A_MN ? 2048 : 32;
       constexpr uint32_t b_lbo = B_MN ? kBK * 128 : 16, b_step = B_MN ? 2048 : 32;
       uint32_t kc = 0, tile = 0;
@@ -159,23 +180,26 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
         int m_blk, split, n0, n1;
         sched.unit(u, m_blk, split, n0, n1);
         for (int nb = n0; ok && nb < n1; ++nb, ++tile) {
-          const uint32_t acc = tile & 1u;
-          const uint32_t aph = (tile >> 1) & 1u;
+          const uint32_t acc = tile % NB;
+          const uint32_t aph = (tile / NB) & 1u;
           if (!mbar_wait(&sm.tempty[acc], aph ^ 1u, timeout_ns, abort)) { ok = false; break; }
           tc_fence_after();
-          const uint32_t d_tmem = tmem_base + acc * kBN;
+          const uint32_t d_tmem = tmem_base + acc * kBN;  // NB = 1: halves at columns 0 and 256
           for (int kb = 0; kb < sched.num_kb; ++kb, ++kc) {
-            const int s = kc % kStages;
-            const uint32_t ph = (kc / kStages) & 1u;
+            const int s = kc % S;
+            const uint32_t ph = (kc / S) & 1u;
             if (!mbar_wait(&sm.full[s], ph, timeout_ns, abort)) { ok = false; break; }
             tc_fence_after();
             const uint32_t a_base = smem_addr(sm.a[s]);
             const uint32_t b_base = smem_addr(sm.b[s]);
 #pragma unroll
             for (int k = 0; k < kBK / 16; ++k) {
-              const uint64_t ad = smem_desc_sw128(a_base + k * a_step, a_lbo, 1024);
               const uint64_t bd = smem_desc_sw128(b_base + k * b_step, b_lbo, 1024);
-              umma_bf16(d_tmem, ad, bd, idesc, (kb | k) != 0 ? 1u : 0u);
+#pragma unroll
+              for (int h = 0; h < HALVES; ++h) {
+                const uint64_t ad = smem_desc_sw128(a_base + h * kTileABytes + k * a_step, a_lbo, 1024);
+                umma_bf16(d_tmem + h * kBN, ad, bd, idesc, (kb | k) != 0 ? 1u : 0u);
+              }
             }
             umma_commit(&sm.empty[s]);  // frees the stage once these MMAs have read it
           }
@@ -194,38 +218,46 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
     // ------------------------------------------------------------------ epilogue
     const int quad = warp & 3;                  // TMEM lanes 32*quad .. 32*quad+31
     const int row_in_tile = quad * 32 + lane;
-    typename Epi::State st;
+    typename Epi::State st[HALVES];             // a thread owns row r of each half
     uint32_t tile = 0;
     bool ok = true;
     for (int u = blockIdx.x; ok && u < sched.num_units; u += gridDim.x) {
       int m_blk, split, n0, n1;
       sched.unit(u, m_blk, split, n0, n1);
-      const int row = m_blk * kBM + row_in_tile;
-      Epi::begin_unit(ep, st, row, split);
+      const int row0 = m_blk * Cfg::kRows + row_in_tile;
+#pragma unroll
+      for (int h = 0; h < HALVES; ++h) Epi::begin_unit(ep, st[h], row0 + h * kBM, split);
       for (int nb = n0; nb < n1; ++nb, ++tile) {
-        const uint32_t acc = tile & 1u;
-        const uint32_t aph = (tile >> 1) & 1u;
+        const uint32_t acc = tile % NB;
+        const uint32_t aph = (tile / NB) & 1u;
         // one lane waits; the warp follows it, so tcgen05.ld always runs on a converged warp
         int got = 0;
         if (lane == 0) got = mbar_wait(&sm.tfull[acc], aph, timeout_ns, abort) ? 1 : 0;
         got = __shfl_sync(0xffffffffu, got, 0);
         if (!got) { ok = false; break; }
         tc_fence_after();
-        const uint32_t t_row = tmem_base + (static_cast<uint32_t>(quad * 32) << 16) + acc * kBN;
+#pragma unroll
+        for (int h = 0; h < HALVES; ++h) {
+          const int row = row0 + h * kBM;
+          const uint32_t t_row = tmem_base + (static_cast<uint32_t>(quad * 32) << 16) + acc * kBN + h * kBN;
 #pragma unroll 1
-        for (int c = 0; c < kBN / 32; ++c) {
-          uint32_t r[32];
-          tmem_ld32(t_row + c * 32, r);
-          tmem_ld_wait();
-          if (c == kBN / 32 - 1) {
-            // the accumulator has been read completely: hand it back to the MMA warp
-            tc_fence_before();
-            mbar_arrive(&sm.tempty[acc]);
+          for (int c = 0; c < kBN / 32; ++c) {
+            uint32_t r[32];
+            tmem_ld32(t_row + c * 32, r);
+            tmem_ld_wait();
+            if (h == HALVES - 1 && c == kBN / 32 - 1) {
+              // the accumulator has been read completely: hand it back to the MMA warp
+              tc_fence_before();
+              mbar_arrive(&sm.tempty[acc]);
+            }
+            Epi::chunk(ep, st[h], row, nb * kBN + c * 32, r);
           }
-          Epi::chunk(ep, st, row, nb * kBN + c * 32, r);
         }
       }
-      if (ok) Epi::end_unit(ep, st, row, split);
+      if (ok) {
+#pragma unroll
+        for (int h = 0; h < HALVES; ++h) Epi::end_unit(ep, st[h], row0 + h * kBM, split);
+      }
     }
     if (!ok) {
       *abort = 1;
@@ -240,7 +272,6 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
     tmem_dealloc(tmem_base, kTmemCols);
   }
 }
-
 
 // =============================================================================================
 // CTA-pair variant (tcgen05 cta_group::2). A cluster of two CTAs computes 256 x 256 output
