@@ -149,6 +149,12 @@ int ps_pack_prefixes(int P, int K, int T_max, int d, int dtype,
  * adv, w [N] f32. Outputs: loss [1] f64 (device), lse, logp, ratio, coef [N] f32,
  * row_loss [N] f32 (may be NULL). Only O(N) values are written; the N x V logits
  * are never stored.
+ * Workspace: ps_lmhead_ppo_fwd_workspace_size() bytes hold one (max, sum) partial per row
+ * for every 256-column vocabulary tile (bf16: 8 B x ceil(V/256) per row, plus 4 B per row
+ * and a few KB), the fastest schedule. A smaller bf16 workspace is accepted down to one
+ * partial per row; the forward then splits the vocabulary into as many ranges as fit
+ * (more passes over W). f32 needs the full size. Too small: PS_ERR_WORKSPACE, nothing
+ * launched.
  * Limits: N >= 0 (N = 0 writes loss = 0), 1 <= V < 2^31, d % 8 == 0 (bf16) or
  * d % 4 == 0 (f32); 16-byte aligned Hpk and W.
  * ------------------------------------------------------------------------- */
@@ -192,9 +198,11 @@ int ps_lmhead_ppo_bwd(int64_t N, int d, int V, int dtype, const void* Hpk, const
  * library routine).
  *  - Memory: every GPU that loads the library holds the 64 MiB array until the
  *    process exits.
- *  - Limit: the problem's workspace (ps_lmhead_ppo_fwd_workspace_size) must fit in
- *    64 MiB: about N <= 508,000 packed rows for bf16; for f32, N * ceil(V/64) * 8
- *    bytes must fit. Larger problems return PS_ERR_UNSUPPORTED and launch nothing.
+ *  - Limit: the forward takes as many vocabulary partials per row as 64 MiB hold. For bf16
+ *    it needs at least one (12 bytes per packed row plus a few KB: about 5.5 million rows);
+ *    all ceil(V/256) of them, the fastest schedule, fit up to about 14,000 rows at
+ *    V = 152064. For f32, N * ceil(V/64) * 8 bytes must fit. Larger problems return
+ *    PS_ERR_UNSUPPORTED and launch nothing.
  *  - Set-up: the first call on each device looks up the array's device address
  *    (cudaGetSymbolAddress) with that device current; make that first call before
  *    any stream capture.

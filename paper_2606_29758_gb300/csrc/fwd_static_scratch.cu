@@ -46,13 +46,14 @@ extern "C" int ps_lmhead_ppo_fwd_noalloc(int64_t N, int d, int V, int dtype, con
                                          const float* w, double eps, double loss_scale, double* loss, float* lse,
                                          float* logp, float* ratio, float* coef, float* row_loss,
                                          ps_stream_t stream) {
-  const size_t need = ps_lmhead_ppo_fwd_workspace_size(N, d, V, dtype);
-  if (need == 0) return PS_ERR_INVALID_ARG;
-  if (need > kStaticScratchBytes) return PS_ERR_UNSUPPORTED;  // problem larger than the static scratch
+  if (ps_lmhead_ppo_fwd_workspace_size(N, d, V, dtype) == 0) return PS_ERR_INVALID_ARG;
   void* scratch = nullptr;
   const int rc = scratch_for_current_device(&scratch);
   if (rc != PS_OK) return rc;
-  // The workspace status word at the head of the scratch is cleared by the call itself.
-  return ps_lmhead_ppo_fwd(N, d, V, dtype, Hpk, W, tok, oldlogp, adv, w, eps, loss_scale, loss, lse, logp, ratio,
-                           coef, row_loss, scratch, kStaticScratchBytes, stream);
+  // The forward takes as many vocabulary partials as the 64 MiB hold; when not even one per row
+  // fits it refuses the workspace before launching anything: the problem is too large for the
+  // static scratch. The status word at the head of the scratch is cleared by the call itself.
+  const int r = ps_lmhead_ppo_fwd(N, d, V, dtype, Hpk, W, tok, oldlogp, adv, w, eps, loss_scale, loss, lse, logp,
+                                  ratio, coef, row_loss, scratch, kStaticScratchBytes, stream);
+  return r == PS_ERR_WORKSPACE ? PS_ERR_UNSUPPORTED : r;
 }

@@ -11,8 +11,9 @@ int device_is_sm103();
 
 // Forward GEMM with the online-logsumexp epilogue. part: [splits][N] (max2, sum) pairs
 // (max in log2 units); ztok: [N] chosen-token logit.
-int max_fwd_splits_bf16();
-int choose_fwd_splits_bf16(int64_t N, int d, int V, int num_sms);
+int fwd_tile_splits_bf16(int V);   // one partial per 256-column vocabulary tile
+// Vocabulary ranges per row block, at most max_splits (the partials the workspace holds).
+int choose_fwd_splits_bf16(int64_t N, int d, int V, int num_sms, int max_splits);
 int fwd_gemm_bf16(int64_t N, int d, int V, const void* Hpk, const void* W, const int32_t* tok, float2* part,
                   float* ztok, int splits, uint32_t* status, cudaStream_t s);
 int fwd_splits_f32(int V);

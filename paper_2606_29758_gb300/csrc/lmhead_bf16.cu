@@ -283,19 +283,18 @@ static int launch_gemm(bool pair, const CUtensorMap& ta, const CUtensorMap& tb, 
               : launch_gemm_single<A_MN, B_MN, Epi>(ta, tb, M, N, K, splits, band_m, ep, status, s);
 }
 
-constexpr int kMaxFwdSplits = 16;
-int max_fwd_splits_bf16() { return kMaxFwdSplits; }
+int fwd_tile_splits_bf16(int V) { return (V + kBN - 1) / kBN; }
 
-// Pick the number of vocabulary ranges per row block: the makespan of a static round-robin
-// over `workers` (CTAs or CTA pairs), in tiles, is rounds x tiles per unit. Among the split
+// Pick the number of vocabulary ranges per row block (at most max_splits): the makespan of a
+// static round-robin over `workers`, in tiles, is rounds x tiles per unit. Among the split
 // counts within 1% of the best makespan, take the smallest: fewer ranges mean wider bands of
 // row blocks and fewer passes over W.
-static int choose_splits(int64_t m_blocks, int64_t n_blocks, int workers, int min_splits = 1) {
+static int choose_splits(int64_t m_blocks, int64_t n_blocks, int workers, int min_splits, int max_splits) {
   auto cost = [&](int s) {
     const int64_t units = m_blocks * s;
     return ((units + workers - 1) / workers) * ((n_blocks + s - 1) / s);
   };
-  const int hi = static_cast<int>(n_blocks < kMaxFwdSplits ? n_blocks : kMaxFwdSplits);
+  const int hi = static_cast<int>(n_blocks < max_splits ? n_blocks : max_splits);
   if (min_splits > hi) return hi;
   int64_t best = INT64_MAX;
   for (int s = min_splits; s <= hi; ++s) best = cost(s) < best ? cost(s) : best;
@@ -315,30 +314,28 @@ constexpr uint32_t kBRowsBox = kUsePairs ? 128 : kBN;
 constexpr int kFwdHalves = 2;
 constexpr int kRecHalves = 1;
 
-// The forward keeps one band of row blocks in flight; every CTA of the band sweeps its
-// vocabulary range and re-reads its row block for every vocabulary tile, so the band's
-// hidden rows must stay in L2 (129 MB) next to the W tiles being streamed. Cap them at a
-// third of L2; that sets the minimum number of vocabulary ranges per row block.
+// The forward keeps one band of row blocks in flight; every CTA re-reads its row block for
+// every vocabulary tile, so the band's hidden rows must stay in L2 (129 MB) next to the W
+// tiles being streamed: they get a third of it.
 constexpr double kFwdBandL2Bytes = 43e6;
 
-static int fwd_min_splits(int d, int workers);
-
-int choose_fwd_splits_bf16(int64_t N, int d, int V, int num_sms) {
-  const int64_t nb = (V + kBN - 1) / kBN;
-  const int rows = kUsePairs ? 256 : kBM * kFwdHalves;
-  const int workers = kUsePairs ? num_sms / 2 : num_sms;
-  int lo = fwd_min_splits(d, workers);
-  if (lo > nb) lo = static_cast<int>(nb);
-  if (lo > kMaxFwdSplits) lo = kMaxFwdSplits;
-  return choose_splits((N + rows - 1) / rows, nb, workers, lo);
+static int fwd_band_max(int d) {
+  const double block_bytes = static_cast<double>(kBM * kFwdHalves) * d * 2.0;
+  const int b = static_cast<int>(kFwdBandL2Bytes / block_bytes);
+  return b < 1 ? 1 : b;
 }
 
-static int fwd_min_splits(int d, int workers) {
-  const int rows = kUsePairs ? 256 : kBM * kFwdHalves;
-  const double block_bytes = static_cast<double>(rows) * d * 2.0;
-  int band_max = static_cast<int>(kFwdBandL2Bytes / block_bytes);
-  if (band_max < 1) band_max = 1;
-  return (workers + band_max - 1) / band_max;
+// With a partial per vocabulary tile (splits = tiles) every unit is one tile and the band of
+// row blocks walks the vocabulary in lockstep, tile by tile. With fewer partials, units are
+// contiguous vocabulary ranges, and the number of ranges is at least what keeps the band in
+// its L2 share.
+int choose_fwd_splits_bf16(int64_t N, int d, int V, int num_sms, int max_splits) {
+  const int nb = fwd_tile_splits_bf16(V);
+  if (max_splits >= nb) return nb;
+  const int rows = kBM * kFwdHalves;
+  int lo = (num_sms + fwd_band_max(d) - 1) / fwd_band_max(d);
+  if (lo > max_splits) lo = max_splits;
+  return choose_splits((N + rows - 1) / rows, nb, num_sms, lo, max_splits);
 }
 
 int fwd_gemm_bf16(int64_t N, int d, int V, const void* Hpk, const void* W, const int32_t* tok, float2* part,
@@ -349,7 +346,7 @@ int fwd_gemm_bf16(int64_t N, int d, int V, const void* Hpk, const void* W, const
     return PS_ERR_INVALID_ARG;
   FwdLseEpi::Params ep{tok, static_cast<int>(N), V, part, ztok};
   const int workers = num_sms_current();
-  const int band = (workers + splits - 1) / splits;
+  const int band = splits == fwd_tile_splits_bf16(V) ? fwd_band_max(d) : (workers + splits - 1) / splits;
   return launch_gemm_single<false, false, FwdLseEpi, kFwdHalves>(ta, tb, N, V, d, splits, band, ep, status, s);
 }
 

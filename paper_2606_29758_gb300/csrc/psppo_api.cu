@@ -5,6 +5,9 @@
 #include <math.h>
 #include <stdint.h>
 
+#include <climits>
+#include <cstdint>
+
 #include "internal.h"
 #include "ps_common.cuh"
 #include "psppo.h"
@@ -380,29 +383,45 @@ __global__ void __launch_bounds__(1024) loss_reduce_kernel(int64_t nblocks, cons
   }
 }
 
-// Forward workspace: header | part [splits][N] float2 | ztok [N] f32 | block_loss [nb] f64
+// Forward workspace: header | ztok [N] f32 | block_loss [nb] f64 | part [S][N] float2. The
+// (max, sum of exp) partials come last: S, the number of vocabulary ranges per row, is as many
+// as the workspace holds, up to one per 256-column vocabulary tile (bf16) -- at that count every
+// unit of the forward GEMM is one tile, the schedule that keeps W traffic lowest. f32 always
+// uses one partial per 64-column tile.
 struct FwdWs {
   float2* part;
   float* ztok;
   double* block_loss;
-  size_t bytes;
+  int splits;       // S that fits (0 if not even one)
+  size_t bytes;     // bytes used with that S
 };
-static int fwd_splits(int64_t N, int V, int dtype) {
-  return dtype == PS_DTYPE_BF16 ? max_fwd_splits_bf16() : fwd_splits_f32(V);
+static int fwd_full_splits(int V, int dtype) {
+  return dtype == PS_DTYPE_BF16 ? fwd_tile_splits_bf16(V) : fwd_splits_f32(V);
 }
-static FwdWs fwd_ws(void* ws, int64_t N, int V, int dtype) {
-  const int S = fwd_splits(N, V, dtype);
+static size_t fwd_fixed_bytes(int64_t N) {
   const int64_t nb = (N + kFinThreads - 1) / kFinThreads;
-  uint8_t* base = static_cast<uint8_t*>(ws) + kWsHeader;
+  return kWsHeader + align_up(sizeof(float) * N, 256) + align_up(sizeof(double) * (nb > 0 ? nb : 1), 256);
+}
+// the partials are the last region: no padding after them, so S partials need exactly this much
+static size_t fwd_part_bytes(int64_t N, int S) { return sizeof(float2) * static_cast<size_t>(S) * N; }
+// Layout for a workspace of ws_bytes (SIZE_MAX: the full-size layout).
+static FwdWs fwd_ws(void* ws, int64_t N, int V, int dtype, size_t ws_bytes) {
+  const int full = fwd_full_splits(V, dtype);
+  const size_t fixed = fwd_fixed_bytes(N);
   FwdWs f;
-  size_t off = 0;
-  f.part = reinterpret_cast<float2*>(base + off);
-  off += align_up(sizeof(float2) * static_cast<size_t>(S) * N, 256);
-  f.ztok = reinterpret_cast<float*>(base + off);
-  off += align_up(sizeof(float) * N, 256);
-  f.block_loss = reinterpret_cast<double*>(base + off);
-  off += align_up(sizeof(double) * (nb > 0 ? nb : 1), 256);
-  f.bytes = kWsHeader + off;
+  uint8_t* base = static_cast<uint8_t*>(ws);
+  f.ztok = reinterpret_cast<float*>(base + kWsHeader);
+  f.block_loss = reinterpret_cast<double*>(base + kWsHeader + align_up(sizeof(float) * N, 256));
+  f.part = reinterpret_cast<float2*>(base + fixed);
+  int S = full;
+  if (ws_bytes != SIZE_MAX && N > 0) {
+    const size_t room = ws_bytes > fixed ? ws_bytes - fixed : 0;
+    const size_t fit = room / (sizeof(float2) * static_cast<size_t>(N));
+    if (fit < static_cast<size_t>(S)) S = static_cast<int>(fit);
+    if (dtype != PS_DTYPE_BF16 && S < full) S = 0;   // the f32 kernel needs every partial
+  }
+  f.splits = S;
+  f.bytes = fixed + fwd_part_bytes(N, S > 0 ? S : 1);
   return f;
 }
 
@@ -511,7 +530,7 @@ int ps_pack_prefixes(int P, int K, int T_max, int d, int dtype, const int32_t* L
 size_t ps_lmhead_ppo_fwd_workspace_size(int64_t N, int d, int V, int dtype) {
   if (N < 0 || V < 1 || !dtype_ok(dtype)) return 0;
   (void)d;
-  return fwd_ws(nullptr, N, V, dtype).bytes;
+  return fwd_ws(nullptr, N, V, dtype, SIZE_MAX).bytes;
 }
 
 int ps_lmhead_ppo_fwd(int64_t N, int d, int V, int dtype, const void* Hpk, const void* W, const int32_t* tok,
@@ -525,13 +544,14 @@ int ps_lmhead_ppo_fwd(int64_t N, int d, int V, int dtype, const void* Hpk, const
   if (N > 0 && (!al16(Hpk) || !al16(W))) return PS_ERR_INVALID_ARG;
   if (dtype == PS_DTYPE_BF16 && !device_is_sm103()) return PS_ERR_UNSUPPORTED;
   cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
-  FwdWs f = fwd_ws(ws, N, V, dtype);
+  FwdWs f = fwd_ws(ws, N, V, dtype, ws_bytes);
+  if (N > 0 && f.splits < 1) return PS_ERR_WORKSPACE;
   int rc = begin_call(ws, ws_bytes, f.bytes, s);
   if (rc != PS_OK) return rc;
   if (N == 0) return cudaMemsetAsync(loss, 0, sizeof(double), s) == cudaSuccess ? PS_OK : PS_ERR_CUDA;
   int splits;
   if (dtype == PS_DTYPE_BF16) {
-    splits = choose_fwd_splits_bf16(N, d, V, num_sms_current());
+    splits = choose_fwd_splits_bf16(N, d, V, num_sms_current(), f.splits);
     rc = fwd_gemm_bf16(N, d, V, Hpk, W, tok, f.part, f.ztok, splits, status_word(ws), s);
   } else {
     splits = fwd_splits_f32(V);

@@ -64,3 +64,35 @@ def test_seeds_and_steps_select_the_cutoff_draw():
         check_prefix(cfg, b, g, seed=seed, step=step)
         seen.add(tuple(g["H"]))
     assert len(seen) == 4
+
+
+@pytest.mark.parametrize("name", ["head7b_small", "mid"])
+def test_forward_with_fewer_vocabulary_partials(name):
+    # A workspace that holds only a few (max, sum) partials per row makes the forward split the
+    # vocabulary into that many ranges; the results must agree with the one-partial-per-tile run.
+    import torch
+    from paper_2606_29758_gb300 import _binding as B
+    cfg = get_config(name)
+    b, up = gpu_pass(cfg, grads=False)
+    N = up.N
+    full = B.ps_lmhead_ppo_fwd_workspace_size(N, cfg.d, cfg.V, up.dcode)
+    tiles = (cfg.V + 255) // 256
+    for parts in (1, 3, tiles - 1):
+        small = full - 8 * N * (tiles - parts)   # exactly `parts` partials per row fit
+        ws = torch.zeros(small, dtype=torch.uint8, device="cuda")
+        outs = {k: torch.empty(N, device="cuda") for k in ("lse", "logp", "ratio", "coef", "row_loss")}
+        loss = torch.zeros(1, dtype=torch.float64, device="cuda")
+        D = b.dev
+        B.ps_lmhead_ppo_fwd(N, cfg.d, cfg.V, up.dcode, up.hid, D["W"], up.tok, up.oldlogp, up.adv, up.w, cfg.eps,
+                            cfg.loss_scale, loss, outs["lse"], outs["logp"], outs["ratio"], outs["coef"],
+                            outs["row_loss"], ws)
+        torch.cuda.synchronize()
+        assert B.ps_workspace_status(ws)[0] == B.PS_OK
+        assert abs(loss.item() - up.loss.item()) <= 1e-5 * abs(up.loss.item())
+        assert (outs["lse"] - up.lse[:N]).abs().max().item() < 1e-5
+    with pytest.raises(B.PsppoError) as e:
+        tiny_ws = torch.zeros(1024, dtype=torch.uint8, device="cuda")
+        B.ps_lmhead_ppo_fwd(N, cfg.d, cfg.V, up.dcode, up.hid, b.dev["W"], up.tok, up.oldlogp, up.adv, up.w,
+                            cfg.eps, cfg.loss_scale, loss, outs["lse"], outs["logp"], outs["ratio"], outs["coef"],
+                            None, tiny_ws)
+    assert e.value.status == B.PS_ERR_WORKSPACE

@@ -52,8 +52,11 @@ def test_noalloc_forward_matches_workspace_forward_twice(name):
 
 
 def test_noalloc_rejects_problems_larger_than_its_scratch():
+    # 6 million rows need more than 64 MiB even with one partial per row: refused before any launch
+    # (the pointers are valid but never read).
     from paper_2606_29758_gb300 import _binding as B
+    t = torch.zeros(64, device="cuda")
     with pytest.raises(B.PsppoError) as e:
-        B.ps_lmhead_ppo_fwd_noalloc(600_000, 3584, 152064, B.PS_DTYPE_BF16, None, None, None, None, None, None,
-                                    0.2, 1.0, None, None, None, None, None, None)
+        B.ps_lmhead_ppo_fwd_noalloc(6_000_000, 3584, 152064, B.PS_DTYPE_BF16, t, t, t, t, t, t,
+                                    0.2, 1.0, t, t, t, t, t, t)
     assert e.value.status == B.PS_ERR_UNSUPPORTED
