@@ -14,6 +14,10 @@ selects H = min{h : x < U_p[h]}, and then
 holds exactly. The weight is w_p[t] = 1/xi_t = 2^62 / S_p[t].
 
 In full mode (the untruncated control) H = L and every weight is 1.
+
+In "trunc_zero" mode the masses may sum to less than 2^62: the deficit is Pr(H = 0) (no token of
+the completion is kept; the design of Appendix F allows xi_1 < 1). Then H = 0 when x >= U[T], and
+xi_t = (U[T] - U[t-1]) / 2^62.
 """
 from __future__ import annotations
 
@@ -43,19 +47,28 @@ def xi(q_p: np.ndarray) -> np.ndarray:
     return np.array([s / ONE62 for s in survival(q_p)], dtype=np.float64)
 
 
-def inverse_survival_weights(q_p: np.ndarray) -> np.ndarray:
+def survival_with_zero(q_p: np.ndarray):
+    """Pr(H >= t) * 2^62 = U[T] - U[t-1] for t = 1..T (masses may leave Pr(H = 0) = the deficit)."""
+    U = cumulative_masses(q_p)
+    return [U[-1] - U[t - 1] for t in range(1, len(q_p) + 1)]
+
+
+def inverse_survival_weights(q_p: np.ndarray, allow_zero: bool = False) -> np.ndarray:
     """w[t-1] = 1/xi_t = 2^62 / S[t] in float64 (+inf where S[t] = 0: never reached)."""
     out = np.empty(len(q_p), dtype=np.float64)
-    for i, s in enumerate(survival(q_p)):
+    S = survival_with_zero(q_p) if allow_zero else survival(q_p)
+    for i, s in enumerate(S):
         out[i] = float(ONE62) / float(s) if s > 0 else np.inf
     return out
 
 
-def cutoff_from_uniform(U, x: int) -> int:
-    """H = min{h >= 1 : x < U[h]} for x in [0, 2^62)."""
+def cutoff_from_uniform(U, x: int, allow_zero: bool = False) -> int:
+    """H = min{h >= 1 : x < U[h]} for x in [0, 2^62); 0 if x >= U[T] and allow_zero."""
     for h in range(1, len(U)):
         if x < U[h]:
             return h
+    if allow_zero:
+        return 0
     raise ValueError("masses do not cover x: they must sum to 2^62")
 
 
@@ -77,15 +90,16 @@ def sample_cutoffs(q: np.ndarray, L: np.ndarray, K: int, seed: int, step: int,
         H[:] = L
         n[:] = L
         return H, n, np.ones((P, T_max), dtype=np.float64)
+    zero = mode == "trunc_zero"
     w_tab = np.empty((P, T_max), dtype=np.float64)
     for p in range(P):
         U = cumulative_masses(q[p])
-        if U[-1] != ONE62:
+        if U[-1] > ONE62 or (U[-1] != ONE62 and not zero):
             raise ValueError(f"prompt {p}: masses sum to {U[-1]}, not 2^62")
-        w_tab[p] = inverse_survival_weights(q[p])
+        w_tab[p] = inverse_survival_weights(q[p], allow_zero=zero)
         for j in range(K):
             k = p * K + j
             x = cutoff_uniform62(seed, step, traj_base + k)
-            H[k] = cutoff_from_uniform(U, x)
+            H[k] = cutoff_from_uniform(U, x, allow_zero=zero)
             n[k] = min(int(H[k]), int(L[k]))
     return H, n, w_tab

@@ -1,0 +1,186 @@
+"""Cutoff-distribution design (oracle, float64): score proxy, timestep weights, budgeted
+monotone xi, and the integer masses the sampler takes.
+
+Section 3.3 and Appendix D: the output-head score proxy of a token is
+    gamma_t = ||h_t||^2 (1 - 2 p_t(o_t) + ||p_t||^2),
+the squared Frobenius norm of d log p(o_t) / dW = (e_o - p) h^T.
+Section 3.3 (Eq. wtilde_factorized1): per prompt, gamma_bar_t averages gamma_t over the
+group's rollouts at step t; the timestep weight is w_t = gamma_bar_t * u_t, with u_t the
+reward-uncertainty proxy (an input here).
+Appendix F: minimise sum_t w_t / xi_t subject to sum_t xi_t = B and 1 >= xi_1 >= ... >= xi_T.
+Without monotonicity, xi_t = B sqrt(w_t) / sum_j sqrt(w_j). With it, the optimum is constant on
+contiguous blocks with scores s_m = sqrt(W_m / L_m) and xi_m = B s_m / sum_j L_j s_j; pooling
+adjacent violators (PAV) until the scores are non-increasing gives the monotone optimum. With the
+cap xi <= 1, a prefix of coordinates saturates at 1 and the same solution applies to the rest
+with the budget reduced by the prefix length.
+Section 4 (Baselines): the cutoff variants Uniform, Time prior xi_t = exp(-lambda (t-1)),
+Heuristic (closed form, then the running minimum), and the fixed prefix of length L.
+
+Masses: Pr(H = h) = xi_h - xi_{h+1} (xi_{T+1} = 0) and Pr(H = 0) = 1 - xi_1, quantised to
+integers q_h = floor(Pr(H = h) 2^62); the deficit 2^62 - sum_h q_h is the mass of H = 0.
+"""
+from __future__ import annotations
+
+import math
+
+import numpy as np
+
+ONE62 = 1 << 62
+
+
+# ----------------------------------------------------------------------------- score proxy
+def score_proxy(H, W, tok):
+    """gamma_t and the token log-probability log p_t(o_t) for every row (Appendix D)."""
+    H = np.asarray(H, dtype=np.float64)
+    W = np.asarray(W, dtype=np.float64)
+    tok = np.asarray(tok)
+    gamma = np.empty(len(tok))
+    logp = np.empty(len(tok))
+    for r0 in range(0, len(tok), 128):
+        z = H[r0:r0 + 128] @ W.T
+        m = z.max(axis=1, keepdims=True)
+        e = np.exp(z - m)
+        p = e / e.sum(axis=1, keepdims=True)
+        rows = np.arange(z.shape[0])
+        po = p[rows, tok[r0:r0 + 128]]
+        hn = (H[r0:r0 + 128] ** 2).sum(axis=1)
+        gamma[r0:r0 + 128] = hn * (1.0 - 2.0 * po + (p * p).sum(axis=1))
+        logp[r0:r0 + 128] = np.log(po)
+    return gamma, logp
+
+
+# ----------------------------------------------------------------------------- weights
+def group_mean_by_step(values_full, L, K):
+    """gamma_bar[p][t-1] = (1/K) sum over the group's completions that reach step t.
+
+    Completions shorter than t contribute 0 (their score at t is zero): the average is over all
+    K rollouts. values_full is laid out completion after completion (unpacked batch order).
+    Sums run sequentially over k in float64.
+    """
+    L = np.asarray(L)
+    B = len(L)
+    P = B // K
+    T_max = int(L.max())
+    off = np.concatenate([[0], np.cumsum(L)])
+    out = np.zeros((P, T_max))
+    for p in range(P):
+        acc = [0.0] * T_max
+        for j in range(K):
+            k = p * K + j
+            seg = values_full[off[k]:off[k] + L[k]]
+            for t in range(int(L[k])):
+                acc[t] = acc[t] + float(seg[t])
+        out[p] = [a / K for a in acc]
+    return out
+
+
+# ----------------------------------------------------------------------------- design
+def closed_form(w, B):
+    """Unconstrained optimum xi_t = B sqrt(w_t) / sum_j sqrt(w_j) (Appendix F)."""
+    r = [math.sqrt(float(x)) for x in w]
+    tot = 0.0
+    for x in r:
+        tot += x
+    return np.array([B * x / tot for x in r])
+
+
+def pav_blocks(w):
+    """Pool adjacent violators: blocks (start, length, W) whose scores sqrt(W / L) are non-increasing.
+
+    Blocks are pushed left to right; while the last block's score is above the one before it
+    (a violation of xi_1 >= xi_2 >= ...), the two are merged.
+    """
+    blocks = []  # [start, length, weight sum]
+    for t, x in enumerate(w):
+        blocks.append([t, 1, float(x)])
+        while len(blocks) > 1 and math.sqrt(blocks[-2][2] / blocks[-2][1]) < math.sqrt(blocks[-1][2] / blocks[-1][1]):
+            s, n, Wm = blocks.pop()
+            blocks[-1][1] += n
+            blocks[-1][2] += Wm
+    return blocks
+
+
+def monotone_design(w, B):
+    """Monotone optimum without the cap: xi on PAV blocks, xi_m = B s_m / sum_j L_j s_j."""
+    blocks = pav_blocks(w)
+    s = [math.sqrt(Wm / n) for _, n, Wm in blocks]
+    den = 0.0
+    for (_, n, _), sm in zip(blocks, s):
+        den += n * sm
+    xi = np.empty(len(w))
+    for (t0, n, _), sm in zip(blocks, s):
+        xi[t0:t0 + n] = B * sm / den
+    return xi
+
+
+def capped_monotone_design(w, B):
+    """Monotone optimum with xi <= 1: the smallest saturated prefix p for which the design of the
+    suffix with budget B - p starts at or below 1 (Appendix F, remark on the cap)."""
+    T = len(w)
+    if not (0 < B <= T):
+        raise ValueError("the budget must lie in (0, T]")
+    for p in range(T):
+        rest = monotone_design(w[p:], B - p)
+        if rest[0] <= 1.0:
+            return np.concatenate([np.ones(p), rest])
+    return np.ones(T)
+
+
+def heuristic_design(w, B):
+    """Section 4 (Heuristic): closed form, then xi_t <- min(xi_{t-1}, xi_t); capped at 1."""
+    xi = closed_form(w, B)
+    for t in range(1, len(xi)):
+        xi[t] = min(xi[t - 1], xi[t])
+    return np.minimum(xi, 1.0)
+
+
+def time_prior_design(T, B, iters=200):
+    """Section 4 (Time prior): xi_t = exp(-lam (t-1)), with lam >= 0 chosen so sum_t xi_t = B."""
+    if not (0 < B <= T):
+        raise ValueError("the budget must lie in (0, T]")
+    t = np.arange(T, dtype=np.float64)
+
+    def budget(lam):
+        return float(np.exp(-lam * t).sum())
+
+    if budget(0.0) <= B:
+        return np.ones(T)
+    lo, hi = 0.0, 1.0
+    while budget(hi) > B:
+        hi *= 2.0
+    for _ in range(iters):
+        mid = 0.5 * (lo + hi)
+        if budget(mid) > B:
+            lo = mid
+        else:
+            hi = mid
+    return np.exp(-hi * t)
+
+
+def uniform_design(T):
+    """Section 4 (Uniform): the cutoff is uniform on 1..T, so xi_t = (T - t + 1) / T."""
+    return (T - np.arange(T, dtype=np.float64)) / T
+
+
+def fixed_prefix_design(T, Lfix):
+    """Section 4 (fixed prefix): H = min(Lfix, T) with probability 1 (biased control)."""
+    return (np.arange(1, T + 1) <= Lfix).astype(np.float64)
+
+
+def masses_from_xi(xi):
+    """Integer masses q_h = floor((xi_h - xi_{h+1}) 2^62), h = 1..T; the deficit is Pr(H = 0).
+
+    Rounding can make the differences add up to slightly more than xi_1; any excess over 2^62
+    (only possible when xi_1 is 1) is taken from the largest mass, lowest index on ties.
+    """
+    T = len(xi)
+    q = [0] * T
+    for h in range(T):
+        nxt = float(xi[h + 1]) if h + 1 < T else 0.0
+        d = float(xi[h]) - nxt
+        q[h] = int(math.floor(d * float(ONE62))) if d > 0.0 else 0
+    excess = sum(q) - ONE62
+    if excess > 0:
+        i = max(range(T), key=lambda j: (q[j], -j))
+        q[i] -= excess
+    return np.array(q, dtype=np.uint64)

@@ -1,0 +1,153 @@
+"""Pins for the oracle's cutoff design (Section 3.3, Appendices D and F, Section 4 variants)."""
+import math
+
+import numpy as np
+import pytest
+from scipy.optimize import minimize
+
+from oracle import design
+from oracle.cutoffs import ONE62, cumulative_masses, inverse_survival_weights, sample_cutoffs
+
+
+def _objective(w, xi):
+    return float(np.sum(np.asarray(w) / np.asarray(xi)))
+
+
+def _brute(w, B, cap):
+    """The design problem solved by a general constrained solver (SLSQP). Monotonicity holds by
+    construction: xi_t = sum_{j >= t} y_j with y >= 0."""
+    T = len(w)
+    to_xi = lambda y: np.cumsum(y[::-1])[::-1]  # noqa: E731
+    cons = [{"type": "eq", "fun": lambda y: np.sum(to_xi(y)) - B}]
+    if cap:
+        cons.append({"type": "ineq", "fun": lambda y: 1.0 - np.sum(y)})
+    best = None
+    for start_xi in (np.full(T, B / T), np.linspace(1.6, 0.4, T) * B / T, np.linspace(1.2, 0.8, T) * B / T):
+        if cap:
+            start_xi = np.minimum(start_xi, 1.0)
+        y0 = np.maximum(np.append(-np.diff(start_xi), start_xi[-1]), 1e-6)
+        for method, opts in (("SLSQP", {"ftol": 1e-15, "maxiter": 5000}),
+                             ("trust-constr", {"xtol": 1e-14, "gtol": 1e-12, "maxiter": 20000})):
+            r = minimize(lambda y: _objective(w, to_xi(y)), y0, method=method, bounds=[(1e-12, None)] * T,
+                         constraints=cons, options=opts)
+            feasible = abs(np.sum(to_xi(r.x)) - B) < 1e-9 and np.all(r.x >= -1e-12) and \
+                (not cap or np.sum(r.x) <= 1.0 + 1e-9)
+            if feasible and (best is None or r.fun < best.fun):    # SLSQP's success flag is often
+                best = r                                            # spuriously false at the optimum
+    assert best is not None
+    best.x = to_xi(best.x)
+    return best
+
+
+@pytest.mark.parametrize("seed", range(8))
+def test_pav_matches_a_general_solver(seed):
+    rng = np.random.default_rng(seed)
+    T = int(rng.integers(3, 8))
+    w = rng.uniform(0.05, 3.0, T) ** 2
+    B = float(rng.uniform(0.3, 0.9) * T) if seed % 2 else float(rng.uniform(0.1, 0.4) * T)
+    xi = design.monotone_design(w, B)
+    assert np.all(np.diff(xi) <= 1e-15) and abs(xi.sum() - B) < 1e-12
+    ref = _brute(w, B, cap=False)
+    assert _objective(w, xi) <= ref.fun * (1 + 1e-7)
+    np.testing.assert_allclose(xi, ref.x, rtol=2e-4, atol=2e-5)
+
+
+@pytest.mark.parametrize("seed", range(6))
+def test_capped_design_matches_a_general_solver(seed):
+    rng = np.random.default_rng(100 + seed)
+    T = int(rng.integers(3, 8))
+    w = np.sort(rng.uniform(0.1, 4.0, T))[::-1] ** 3          # steep front weights force saturation
+    w[rng.integers(0, T)] *= 5.0                               # plus a violation to pool
+    B = float(rng.uniform(0.6, 0.95) * T)
+    xi = design.capped_monotone_design(w, B)
+    assert np.all(xi <= 1.0 + 1e-15) and np.all(np.diff(xi) <= 1e-15) and abs(xi.sum() - B) < 1e-12
+    ref = _brute(w, B, cap=True)
+    assert _objective(w, xi) <= ref.fun * (1 + 1e-7)
+    np.testing.assert_allclose(xi, ref.x, rtol=2e-4, atol=2e-5)
+
+
+def test_closed_form_special_cases():
+    # already non-increasing sqrt(w): no pooling, the unconstrained closed form is the answer
+    w = np.array([9.0, 4.0, 4.0, 1.0])
+    np.testing.assert_allclose(design.monotone_design(w, 2.0), 2.0 * np.sqrt(w) / np.sqrt(w).sum(), rtol=1e-15)
+    np.testing.assert_allclose(design.closed_form(w, 2.0), [2 * 3 / 8, 2 * 2 / 8, 2 * 2 / 8, 2 * 1 / 8])
+    # increasing weights pool into one block: uniform xi = B / T
+    np.testing.assert_allclose(design.monotone_design(np.array([1.0, 2.0, 3.0, 4.0]), 2.0), 0.5, rtol=1e-15)
+    # a single violating pair pools to sqrt of its mean weight
+    xi = design.monotone_design(np.array([4.0, 1.0, 9.0]), 1.0)
+    s = [2.0, math.sqrt(5.0), math.sqrt(5.0)]     # blocks [4] | [1, 9] -> 2 < sqrt(5): all pool
+    assert xi[0] == pytest.approx(xi[1]) == pytest.approx(xi[2])
+    assert s[0] < s[1]
+
+
+def test_time_prior_and_uniform_and_fixed():
+    xi = design.time_prior_design(500, 64.0)
+    assert abs(xi.sum() - 64.0) < 1e-9 and xi[0] == 1.0 and np.all(np.diff(xi) < 0)
+    lam = -math.log(xi[1])
+    np.testing.assert_allclose(xi, np.exp(-lam * np.arange(500)), rtol=1e-12)
+    u = design.uniform_design(10)
+    assert u[0] == 1.0 and u[-1] == pytest.approx(0.1) and u.sum() == pytest.approx(5.5)   # E[H] = (T+1)/2
+    f = design.fixed_prefix_design(10, 4)
+    assert list(f) == [1, 1, 1, 1, 0, 0, 0, 0, 0, 0]
+    h = design.heuristic_design(np.array([1.0, 4.0, 0.25, 1.0]), 2.0)
+    assert np.all(np.diff(h) <= 0) and np.all(h <= 1.0)
+
+
+def test_masses_realise_xi_and_the_budget():
+    rng = np.random.default_rng(3)
+    w = rng.uniform(0.1, 2.0, 300) ** 2
+    xi = design.capped_monotone_design(w, 40.0)
+    q = design.masses_from_xi(xi)
+    U = cumulative_masses(q)
+    assert U[-1] <= ONE62
+    # Pr(H = 0) = 1 - xi_1; Pr(H >= t) = xi_t up to the 2^-62 quantisation; E[H] = sum xi = B
+    assert abs((ONE62 - U[-1]) / ONE62 - (1.0 - xi[0])) < 1e-15 * 300
+    real = np.array([(U[-1] - U[t - 1]) / ONE62 for t in range(1, 301)])
+    np.testing.assert_allclose(real, xi, rtol=1e-12, atol=1e-15 * 300)
+    EH = sum((h + 1) * int(m) for h, m in enumerate(q)) / ONE62
+    assert EH == pytest.approx(40.0, rel=1e-12)
+
+
+def test_zero_cutoff_mode_draws_h0_with_the_deficit():
+    T, M = 12, 4000
+    xi = design.monotone_design(np.ones(T), 3.0)          # uniform xi = 0.25
+    q = design.masses_from_xi(xi)[None]
+    L = np.full(1, T, dtype=np.int32)
+    Hs = np.array([sample_cutoffs(q, L, 1, seed=1, step=s, mode="trunc_zero")[0][0] for s in range(M)])
+    p0 = (Hs == 0).mean()
+    assert abs(p0 - 0.75) < 4.5 * math.sqrt(0.75 * 0.25 / M)
+    w = inverse_survival_weights(q[0], allow_zero=True)
+    np.testing.assert_allclose(w, 4.0, rtol=1e-12)
+    with pytest.raises(ValueError):
+        sample_cutoffs(q, L, 1, seed=1, step=0, mode="trunc")    # the exact mode insists on 2^62
+
+
+def test_group_mean_by_step_by_hand():
+    L = np.array([3, 1, 2, 2])
+    vals = np.array([1., 2., 3., 10., 5., 6., 7., 8.])
+    g = design.group_mean_by_step(vals, L, 2)
+    np.testing.assert_allclose(g, [[(1 + 10) / 2, 2 / 2, 3 / 2], [(5 + 7) / 2, (6 + 8) / 2, 0.0]])
+
+
+def test_score_proxy_is_the_squared_head_gradient_norm():
+    # gamma = || d log p(o) / dW ||_F^2, checked by central differences over every entry of W
+    rng = np.random.default_rng(7)
+    d, V = 3, 5
+    H = rng.standard_normal((4, d))
+    W = rng.standard_normal((V, d)) * 0.7
+    tok = np.array([0, 4, 2, 2])
+    gamma, logp = design.score_proxy(H, W, tok)
+    eps = 1e-6
+    for i in range(4):
+        def lp(Wm):
+            z = Wm @ H[i]
+            return z[tok[i]] - (z.max() + math.log(np.exp(z - z.max()).sum()))
+        g = np.zeros_like(W)
+        for v in range(V):
+            for c in range(d):
+                Wp, Wn = W.copy(), W.copy()
+                Wp[v, c] += eps
+                Wn[v, c] -= eps
+                g[v, c] = (lp(Wp) - lp(Wn)) / (2 * eps)
+        assert gamma[i] == pytest.approx(float((g * g).sum()), rel=1e-7)
+        assert logp[i] == pytest.approx(lp(W), rel=1e-13)
