@@ -48,7 +48,7 @@ typedef enum {
   PS_ERR_CUDA = 7           /* a CUDA runtime call failed */
 } ps_status;
 
-enum { PS_MODE_TRUNC = 0, PS_MODE_FULL = 1 };
+enum { PS_MODE_TRUNC = 0, PS_MODE_FULL = 1, PS_MODE_TRUNC_ZERO = 2 };
 enum { PS_DTYPE_BF16 = 0, PS_DTYPE_F32 = 1 };
 enum { PS_ADV_CENTERED = 0, PS_ADV_GROUP_NORM = 1 };
 enum { PS_DW_OVERWRITE = 0, PS_DW_ACCUMULATE = 1 };
@@ -88,7 +88,10 @@ int ps_workspace_status(const void* ws, ps_stream_t stream, uint32_t* bits);
  *        key = (seed, 0x5053505030303031))[0]) >> 2, as H = min{h : x < U[h]},
  *        U[h] = q[p][0] + ... + q[p][h-1]. traj_base is the global index of the
  *        first completion, so a batch split across ranks draws the same cutoffs.
- * mode   PS_MODE_TRUNC, or PS_MODE_FULL (H = L, weights 1: the untruncated control).
+ * mode   PS_MODE_TRUNC, PS_MODE_FULL (H = L, weights 1: the untruncated control), or
+ *        PS_MODE_TRUNC_ZERO: the masses may sum to less than 2^62 and the deficit is
+ *        Pr(H = 0) (the design of Appendix F allows xi_1 < 1); a draw x >= U[T] gives H = 0
+ *        and n = 0, and S_p[t] = U_p[T] - U_p[t-1]. A sum above 2^62 sets PS_DEV_BAD_PMF.
  * H, n   [B] int32 outputs: the cutoff and the prefix length n = min(H, L).
  * w_tab  [P][T_max] f32 output: w_tab[p][t-1] = 2^62 / S_p[t] rounded to f32, with
  *        S_p[t] = 2^62 - U_p[t-1] (so 1/w = xi_t exactly before rounding); +inf
@@ -184,6 +187,56 @@ int ps_lmhead_ppo_bwd(int64_t N, int d, int V, int dtype, const void* Hpk, const
                       const int32_t* tok, const float* lse, const float* coef,
                       float* dH, float* dW, int flags,
                       void* ws, size_t ws_bytes, ps_stream_t stream);
+
+/* ---------------------------------------------------------------------------
+ * ps_lmhead_score_proxy -- per-token output-head score proxy (cutoff design input).
+ *
+ * Appendix D: for a softmax head the squared norm of the head score is
+ *   gamma_i = ||h_i||^2 (1 - 2 p_i(o_i) + ||p_i||^2),  p_i = softmax(W h_i),
+ * with ||p||^2 = exp(LSE(2z) - 2 LSE(z)) (two logsumexp reductions). One pass of the head
+ * GEMM over the rows (e.g. every token of the rollouts, with the old-policy head) gives
+ * gamma [N] f32 and, if logp is not NULL, log p_i(o_i) [N] f32.
+ * Hrows [N][d] bf16, W [V][d] bf16 (bf16 only: other dtypes return PS_ERR_UNSUPPORTED),
+ * tok [N] int32 (PS_DEV_BAD_TOKEN and NaN outputs for ids outside [0, V)).
+ * Workspace: like the forward, as many vocabulary partials (16 B per row each) as fit, up
+ * to ps_lmhead_score_proxy_workspace_size(); at least one per row.
+ * ------------------------------------------------------------------------- */
+size_t ps_lmhead_score_proxy_workspace_size(int64_t N, int d, int V, int dtype);
+int ps_lmhead_score_proxy(int64_t N, int d, int V, int dtype, const void* Hrows, const void* W,
+                          const int32_t* tok, float* gamma, float* logp,
+                          void* ws, size_t ws_bytes, ps_stream_t stream);
+
+/* ---------------------------------------------------------------------------
+ * ps_design_cutoffs -- the per-prompt cutoff distribution and its integer masses.
+ *
+ * Section 3.3 / Algorithm 1 steps 7-9, Appendix F, and the Section 4 variants. For prompt p
+ * with horizon T_p = max of its group's lengths and budget B_p = min(budget, T_p):
+ *  PS_DESIGN_OPTIMIZED: gamma_bar_t = (1/K) sum of gamma over the group's completions that
+ *    reach step t (shorter ones count as 0); w_t = gamma_bar_t * u_t (u_t = 1 if u is NULL),
+ *    raised to at least 1e-12 * max_t w_t; xi minimises sum_t w_t / xi_t subject to
+ *    sum_t xi_t = B_p and 1 >= xi_1 >= ... >= xi_T_p: pooled blocks with
+ *    xi_m = B s_m / sum_j L_j s_j, s_m = sqrt(W_m / L_m) (adjacent violators merged), and the
+ *    smallest saturated prefix xi = 1 whose remaining design starts at or below 1.
+ *  PS_DESIGN_HEURISTIC: xi_t = B sqrt(w_t) / sum_j sqrt(w_j), then xi_t <- min(xi_{t-1}, xi_t),
+ *    then min(xi_t, 1).
+ *  PS_DESIGN_UNIFORM: xi_t = (T_p - t + 1) / T_p (cutoff uniform on 1..T_p; budget unused).
+ *  PS_DESIGN_TIME_PRIOR: xi_t = exp(-lambda (t - 1)), lambda >= 0 with sum_t xi_t = B_p.
+ *  PS_DESIGN_FIXED: xi_t = 1 for t <= param, 0 after (the biased fixed-prefix control).
+ * Outputs: q [P][T_max] uint64 masses, q[p][h-1] = floor((xi_h - xi_{h+1}) 2^62) (xi_{T+1} = 0;
+ * an excess over 2^62 from rounding is taken off the largest mass), zero beyond T_p; the
+ * deficit 2^62 - sum_h q[p][h-1] is Pr(H = 0): sample with PS_MODE_TRUNC_ZERO. xi [P][T_max]
+ * f64 (may be NULL). Inputs: L [B] int32, gamma_full [sum L] f32 in completion order (needed
+ * by OPTIMIZED and HEURISTIC, may be NULL otherwise), u [P][T_max] f32 or NULL.
+ * All arithmetic is sequential f64, so the masses are reproducible bit for bit.
+ * ------------------------------------------------------------------------- */
+enum {
+  PS_DESIGN_OPTIMIZED = 0, PS_DESIGN_HEURISTIC = 1, PS_DESIGN_UNIFORM = 2,
+  PS_DESIGN_TIME_PRIOR = 3, PS_DESIGN_FIXED = 4
+};
+size_t ps_design_cutoffs_workspace_size(int P, int K, int T_max);
+int ps_design_cutoffs(int P, int K, int T_max, const int32_t* L, const float* gamma_full,
+                      const float* u, double budget, int strategy, double param,
+                      uint64_t* q, double* xi, void* ws, size_t ws_bytes, ps_stream_t stream);
 
 /* ---------------------------------------------------------------------------
  * ps_lmhead_ppo_fwd_noalloc -- ps_lmhead_ppo_fwd for callers that cannot allocate.

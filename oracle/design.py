@@ -30,7 +30,8 @@ ONE62 = 1 << 62
 
 # ----------------------------------------------------------------------------- score proxy
 def score_proxy(H, W, tok):
-    """gamma_t and the token log-probability log p_t(o_t) for every row (Appendix D)."""
+    """gamma_t = ||h_t||^2 ||e_o - p_t||^2 and log p_t(o_t) for every row (Appendix D; the paper's
+    1 - 2 p(o) + ||p||^2 is ||e_o - p||^2 expanded)."""
     H = np.asarray(H, dtype=np.float64)
     W = np.asarray(W, dtype=np.float64)
     tok = np.asarray(tok)
@@ -44,7 +45,9 @@ def score_proxy(H, W, tok):
         rows = np.arange(z.shape[0])
         po = p[rows, tok[r0:r0 + 128]]
         hn = (H[r0:r0 + 128] ** 2).sum(axis=1)
-        gamma[r0:r0 + 128] = hn * (1.0 - 2.0 * po + (p * p).sum(axis=1))
+        resid = -p                                   # e_o - p, written out: no cancellation near p(o) = 1
+        resid[rows, tok[r0:r0 + 128]] += 1.0
+        gamma[r0:r0 + 128] = hn * (resid * resid).sum(axis=1)
         logp[r0:r0 + 128] = np.log(po)
     return gamma, logp
 
@@ -184,3 +187,54 @@ def masses_from_xi(xi):
         i = max(range(T), key=lambda j: (q[j], -j))
         q[i] -= excess
     return np.array(q, dtype=np.uint64)
+
+
+# ----------------------------------------------------------------------------- whole design step
+STRATEGIES = ("optimized", "heuristic", "uniform", "time_prior", "fixed")
+W_FLOOR = 1e-12   # weights below W_FLOOR * max_t w_t are raised to it, so every xi_t > 0
+
+
+def timestep_weights(gamma_bar_p, u_p):
+    """w_t = gamma_bar_t * u_t (u = 1 when not given), floored at W_FLOOR * max_t w_t so that the
+    design keeps xi_t > 0 (Section 3.2 requires xi_T > 0); all-zero weights become all ones."""
+    T = len(gamma_bar_p)
+    w = [float(gamma_bar_p[t]) * (float(u_p[t]) if u_p is not None else 1.0) for t in range(T)]
+    wmax = max(w)
+    if not wmax > 0.0:
+        return [1.0] * T
+    fl = W_FLOOR * wmax
+    return [x if x > fl else fl for x in w]
+
+
+def design_cutoff_masses(L, K, gamma_full, u, B, strategy, param=0.0):
+    """Masses q [P, T_max] (uint64) and xi [P, T_max] (float64) for every prompt.
+
+    Prompt p's horizon is T_p = the longest completion of its group; its budget is min(B, T_p).
+    optimized: capped monotone design of w; heuristic: closed form + running minimum + cap;
+    uniform: xi_t = (T_p - t + 1) / T_p; time_prior: exp(-lam (t-1)) with sum_t xi_t = budget;
+    fixed: xi_t = 1 for t <= param.
+    """
+    L = np.asarray(L)
+    B_total = len(L)
+    P = B_total // K
+    T_max = int(L.max())
+    gbar = group_mean_by_step(gamma_full, L, K) if strategy in ("optimized", "heuristic") else None
+    q = np.zeros((P, T_max), dtype=np.uint64)
+    xi_all = np.zeros((P, T_max))
+    for p in range(P):
+        Tp = int(L[p * K:(p + 1) * K].max())
+        Bp = min(float(B), float(Tp))
+        if strategy in ("optimized", "heuristic"):
+            w = timestep_weights(gbar[p, :Tp], None if u is None else u[p, :Tp])
+            xi = capped_monotone_design(w, Bp) if strategy == "optimized" else heuristic_design(w, Bp)
+        elif strategy == "uniform":
+            xi = uniform_design(Tp)
+        elif strategy == "time_prior":
+            xi = time_prior_design(Tp, Bp)
+        elif strategy == "fixed":
+            xi = fixed_prefix_design(Tp, int(param))
+        else:
+            raise ValueError(strategy)
+        q[p, :Tp] = masses_from_xi(xi)
+        xi_all[p, :Tp] = xi
+    return q, xi_all

@@ -16,7 +16,7 @@ LIB_PATH = os.path.join(_PKG, "libpsppo.so")
 
 PS_OK, PS_ERR_INVALID_ARG, PS_ERR_UNSUPPORTED, PS_ERR_WORKSPACE, PS_ERR_CAPACITY, \
     PS_ERR_DEVICE_DATA, PS_ERR_TIMEOUT, PS_ERR_CUDA = range(8)
-PS_MODE_TRUNC, PS_MODE_FULL = 0, 1
+PS_MODE_TRUNC, PS_MODE_FULL, PS_MODE_TRUNC_ZERO = 0, 1, 2
 PS_DTYPE_BF16, PS_DTYPE_F32 = 0, 1
 PS_ADV_CENTERED, PS_ADV_GROUP_NORM = 0, 1
 PS_DW_OVERWRITE, PS_DW_ACCUMULATE = 0, 1
@@ -29,16 +29,20 @@ EXPORTS = [
     "ps_lmhead_ppo_fwd_workspace_size", "ps_lmhead_ppo_fwd",
     "ps_lmhead_ppo_bwd_workspace_size", "ps_lmhead_ppo_bwd",
     "ps_diag_gemm_bf16", "ps_diag_wait_timeout", "ps_lmhead_ppo_fwd_noalloc",
+    "ps_lmhead_score_proxy_workspace_size", "ps_lmhead_score_proxy",
+    "ps_design_cutoffs_workspace_size", "ps_design_cutoffs",
 ]
+PS_DESIGN_OPTIMIZED, PS_DESIGN_HEURISTIC, PS_DESIGN_UNIFORM, PS_DESIGN_TIME_PRIOR, PS_DESIGN_FIXED = range(5)
 
 
 __all__ = EXPORTS + [
     "PsppoError", "lib", "status_string", "dtype_code", "LIB_PATH",
     "PS_OK", "PS_ERR_INVALID_ARG", "PS_ERR_UNSUPPORTED", "PS_ERR_WORKSPACE", "PS_ERR_CAPACITY",
-    "PS_ERR_DEVICE_DATA", "PS_ERR_TIMEOUT", "PS_ERR_CUDA", "PS_MODE_TRUNC", "PS_MODE_FULL",
+    "PS_ERR_DEVICE_DATA", "PS_ERR_TIMEOUT", "PS_ERR_CUDA", "PS_MODE_TRUNC", "PS_MODE_FULL", "PS_MODE_TRUNC_ZERO",
     "PS_DTYPE_BF16", "PS_DTYPE_F32", "PS_ADV_CENTERED", "PS_ADV_GROUP_NORM", "PS_DW_OVERWRITE",
     "PS_DW_ACCUMULATE", "PS_DEV_BAD_PMF", "PS_DEV_BAD_LENGTH", "PS_DEV_CAPACITY", "PS_DEV_BAD_TOKEN",
-    "PS_DEV_TIMEOUT",
+    "PS_DEV_TIMEOUT", "PS_DESIGN_OPTIMIZED", "PS_DESIGN_HEURISTIC", "PS_DESIGN_UNIFORM",
+    "PS_DESIGN_TIME_PRIOR", "PS_DESIGN_FIXED",
 ]
 
 
@@ -71,6 +75,10 @@ _SIGS = {
     "ps_diag_gemm_bf16": (_i32, [_i32, _i32, _i32, _i32, _i32, _vp, _i64, _vp, _i64, _vp, _i64, _i32, _i32, _vp, _sz,
                                  _vp]),
     "ps_diag_wait_timeout": (_i32, [_u64, _vp, _sz, _vp]),
+    "ps_lmhead_score_proxy_workspace_size": (_sz, [_i64, _i32, _i32, _i32]),
+    "ps_lmhead_score_proxy": (_i32, [_i64, _i32, _i32, _i32, _vp, _vp, _vp, _vp, _vp, _vp, _sz, _vp]),
+    "ps_design_cutoffs_workspace_size": (_sz, [_i32, _i32, _i32]),
+    "ps_design_cutoffs": (_i32, [_i32, _i32, _i32, _vp, _vp, _vp, _f64, _i32, _f64, _vp, _vp, _vp, _sz, _vp]),
     "ps_lmhead_ppo_fwd_noalloc": (_i32, [_i64, _i32, _i32, _i32, _vp, _vp, _vp, _vp, _vp, _vp, _f64, _f64,
                                          _vp, _vp, _vp, _vp, _vp, _vp, _vp]),
 }
@@ -190,6 +198,26 @@ def ps_lmhead_ppo_fwd_noalloc(N, d, V, dtype, Hpk, W, tok, oldlogp, adv, w, eps,
                                          _ptr(w), float(eps), float(loss_scale), _ptr(loss), _ptr(lse), _ptr(logp),
                                          _ptr(ratio), _ptr(coef), _ptr(row_loss), _stream(stream))
     _check(rc, "ps_lmhead_ppo_fwd_noalloc")
+
+
+def ps_lmhead_score_proxy_workspace_size(N: int, d: int, V: int, dtype: int) -> int:
+    return lib().ps_lmhead_score_proxy_workspace_size(N, d, V, dtype)
+
+
+def ps_lmhead_score_proxy(N, d, V, dtype, Hrows, W, tok, gamma, logp, ws, stream=None):
+    rc = lib().ps_lmhead_score_proxy(N, d, V, dtype, _ptr(Hrows), _ptr(W), _ptr(tok), _ptr(gamma), _ptr(logp),
+                                     _ptr(ws), _nbytes(ws), _stream(stream))
+    _check(rc, "ps_lmhead_score_proxy")
+
+
+def ps_design_cutoffs_workspace_size(P: int, K: int, T_max: int) -> int:
+    return lib().ps_design_cutoffs_workspace_size(P, K, T_max)
+
+
+def ps_design_cutoffs(P, K, T_max, L, gamma_full, u, budget, strategy, param, q, xi, ws, stream=None):
+    rc = lib().ps_design_cutoffs(P, K, T_max, _ptr(L), _ptr(gamma_full), _ptr(u), float(budget), int(strategy),
+                                 float(param), _ptr(q), _ptr(xi), _ptr(ws), _nbytes(ws), _stream(stream))
+    _check(rc, "ps_design_cutoffs")
 
 
 def ps_lmhead_ppo_bwd_workspace_size(N: int, d: int, V: int, dtype: int, chunk_rows: int = 0) -> int:

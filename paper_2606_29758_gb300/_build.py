@@ -18,7 +18,7 @@ CSRC = os.path.join(PKG, "csrc")
 INCLUDE = os.path.join(ROOT, "include")
 BUILD = os.path.join(PKG, "_build")
 LIB = os.path.join(PKG, "libpsppo.so")
-SOURCES = ["psppo_api.cu", "lmhead_bf16.cu", "lmhead_f32.cu", "fwd_static_scratch.cu"]
+SOURCES = ["psppo_api.cu", "lmhead_bf16.cu", "lmhead_f32.cu", "fwd_static_scratch.cu", "design.cu"]
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
 
 

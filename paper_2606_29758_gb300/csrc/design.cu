@@ -1,0 +1,387 @@
+// Cutoff-distribution design on the device (the step upstream of the sampler).
+//
+//  ps_lmhead_score_proxy: per token, the output-head score proxy of Appendix D,
+//      gamma = ||h||^2 (1 - 2 p(o) + ||p||^2),
+//  and log p(o), from one pass of the LM-head GEMM (the forward's schedule) whose epilogue keeps
+//  two running exponential sums (||p||^2 from the two-logsumexp identity).
+//  ps_design_cutoffs: per prompt, the group average of gamma at each step (Section 3.3), timestep
+//  weights w = gamma_bar * u, the budgeted monotone xi of Appendix F (closed form + pooling of
+//  adjacent violators + the xi <= 1 cap), or one of the Section 4 variants, and the integer
+//  masses the sampler takes (the deficit is Pr(H = 0)).
+//
+// The design arithmetic is sequential float64 with explicitly rounded operations (no FMA
+// contraction), so the masses are reproducible bit for bit.
+#include <cuda_runtime.h>
+#include <math.h>
+#include <stdint.h>
+
+#include <climits>
+#include <cstdint>
+
+#include "internal.h"
+#include "ps_common.cuh"
+#include "psppo.h"
+
+namespace psk {
+
+static size_t al256(size_t x) { return (x + 255) / 256 * 256; }
+
+// ================================================================== score proxy
+__global__ void row_sqnorm_kernel(int64_t N, int d, int is_bf16, const void* __restrict__ H,
+                                  float* __restrict__ out) {
+  const int lane = threadIdx.x & 31;
+  const int64_t warps = static_cast<int64_t>(gridDim.x) * (blockDim.x >> 5);
+  for (int64_t i = static_cast<int64_t>(blockIdx.x) * (blockDim.x >> 5) + (threadIdx.x >> 5); i < N; i += warps) {
+    float acc = 0.f;
+    if (is_bf16) {
+      const uint4* r = reinterpret_cast<const uint4*>(static_cast<const uint16_t*>(H) + i * d);
+      for (int c = lane; c < d / 8; c += 32) {
+        const uint4 v = r[c];
+        const uint32_t w4[4] = {v.x, v.y, v.z, v.w};
+#pragma unroll
+        for (int k = 0; k < 4; ++k) {
+          const float a = __uint_as_float(w4[k] << 16), b = __uint_as_float(w4[k] & 0xFFFF0000u);
+          acc = fmaf(a, a, fmaf(b, b, acc));
+        }
+      }
+    } else {
+      const float* r = static_cast<const float*>(H) + i * d;
+      for (int c = lane; c < d; c += 32) acc = fmaf(r[c], r[c], acc);
+    }
+#pragma unroll
+    for (int o = 16; o >= 1; o >>= 1) acc += __shfl_xor_sync(0xffffffffu, acc, o);
+    if (lane == 0) out[i] = acc;
+  }
+}
+
+__global__ void proxy_finalize_kernel(int64_t N, int V, int splits, const float4* __restrict__ part,
+                                      const float* __restrict__ ztok, const float* __restrict__ hn,
+                                      const int32_t* __restrict__ tok, float* __restrict__ gamma,
+                                      float* __restrict__ logp, uint32_t* status) {
+  const int64_t i = static_cast<int64_t>(blockIdx.x) * blockDim.x + threadIdx.x;
+  if (i >= N) return;
+  float m = -INFINITY;
+  for (int s = 0; s < splits; ++s) m = fmaxf(m, part[static_cast<int64_t>(s) * N + i].x);
+  double S1 = 0.0, S2 = 0.0;
+  for (int s = 0; s < splits; ++s) {
+    const float4 pr = part[static_cast<int64_t>(s) * N + i];
+    const double f = exp2(static_cast<double>(pr.x) - m);
+    S1 += pr.y * f;
+    S2 += pr.z * f * f;
+  }
+  const int t = tok[i];
+  if (t < 0 || t >= V) {
+    raise_status(status, PS_DEV_BAD_TOKEN);
+    gamma[i] = NAN;
+    if (logp) logp[i] = NAN;
+    return;
+  }
+  // S1, S2: sums over the other columns; e_o = 2^(x_o - m) for the chosen one
+  const double x = static_cast<double>(ztok[i]) * 1.4426950408889634 - m;
+  const double eo = exp2(x);
+  const double tot = eo + S1;
+  gamma[i] = static_cast<float>(static_cast<double>(hn[i]) * ((S1 * S1 + S2) / (tot * tot)));
+  if (logp) logp[i] = static_cast<float>((x - log2(tot)) * 0.6931471805599453);
+}
+
+// ================================================================== design
+struct DesignWs {
+  double* w;       // [P][T_max] weights
+  double* xi;      // [P][T_max]
+  double* bW;      // [P][T_max] PAV block weights
+  int32_t* bn;     // [P][T_max] PAV block lengths
+  int64_t* off;    // [P][K] row offsets of the group's completions
+};
+
+// Monotone design of w[0..T) with budget B into xi (Appendix F): pool adjacent violators while
+// sqrt(W_prev / n_prev) < sqrt(W_last / n_last), then xi_m = B s_m / sum_j n_j s_j.
+__device__ void monotone_design_dev(const double* w, int T, double B, double* xi, double* bW, int32_t* bn) {
+  int nb = 0;
+  for (int t = 0; t < T; ++t) {
+    bW[nb] = w[t];
+    bn[nb] = 1;
+    ++nb;
+    while (nb > 1 && __dsqrt_rn(__ddiv_rn(bW[nb - 2], static_cast<double>(bn[nb - 2]))) <
+                         __dsqrt_rn(__ddiv_rn(bW[nb - 1], static_cast<double>(bn[nb - 1])))) {
+      bn[nb - 2] += bn[nb - 1];
+      bW[nb - 2] = __dadd_rn(bW[nb - 2], bW[nb - 1]);
+      --nb;
+    }
+  }
+  double den = 0.0;
+  for (int m = 0; m < nb; ++m) {
+    const double sm = __dsqrt_rn(__ddiv_rn(bW[m], static_cast<double>(bn[m])));
+    den = __dadd_rn(den, __dmul_rn(static_cast<double>(bn[m]), sm));
+  }
+  int t0 = 0;
+  for (int m = 0; m < nb; ++m) {
+    const double sm = __dsqrt_rn(__ddiv_rn(bW[m], static_cast<double>(bn[m])));
+    const double v = __ddiv_rn(__dmul_rn(B, sm), den);
+    for (int j = 0; j < bn[m]; ++j) xi[t0 + j] = v;
+    t0 += bn[m];
+  }
+}
+
+constexpr int kDesignThreads = 256;
+
+__global__ void __launch_bounds__(kDesignThreads)
+    design_kernel(int K, int T_max, const int32_t* __restrict__ L, const float* __restrict__ gamma,
+                  const float* __restrict__ u, double budget, int strategy, double param, uint64_t* __restrict__ q,
+                  double* __restrict__ xi_out, DesignWs ws, uint32_t* status) {
+  const int p = blockIdx.x;
+  const int tid = threadIdx.x;
+  __shared__ int Tp_s;
+  __shared__ double red_d[kDesignThreads / 32];
+  __shared__ unsigned long long red_u[kDesignThreads / 32];
+  __shared__ unsigned long long red_b[kDesignThreads / 32];
+  __shared__ long long red_l[kDesignThreads / 32];
+  __shared__ int red_i[kDesignThreads / 32];
+  __shared__ double lam_s;
+  const int lane = tid & 31, wid = tid >> 5;
+  double* w = ws.w + static_cast<int64_t>(p) * T_max;
+  double* xi = ws.xi + static_cast<int64_t>(p) * T_max;
+  int64_t* off = ws.off + static_cast<int64_t>(p) * K;
+
+  // horizon of the group, and the row offset of its first completion
+  long long base = 0;
+  for (int k = tid; k < p * K; k += kDesignThreads) base += L[k];
+#pragma unroll
+  for (int o = 16; o >= 1; o >>= 1) base += __shfl_xor_sync(0xffffffffu, base, o);
+  if (lane == 0) red_l[wid] = base;
+  __syncthreads();
+  if (tid == 0) {
+    long long b = 0;
+    for (int i = 0; i < kDesignThreads / 32; ++i) b += red_l[i];
+    int Tp = 0;
+    for (int j = 0; j < K; ++j) {
+      off[j] = b;
+      b += L[p * K + j];
+      Tp = max(Tp, L[p * K + j]);
+    }
+    if (Tp < 1 || Tp > T_max) raise_status(status, PS_DEV_BAD_LENGTH);
+    Tp_s = Tp < 1 ? 1 : (Tp > T_max ? T_max : Tp);
+  }
+  __syncthreads();
+  const int Tp = Tp_s;
+  const double Bp = fmin(budget, static_cast<double>(Tp));
+
+  if (strategy == PS_DESIGN_OPTIMIZED || strategy == PS_DESIGN_HEURISTIC) {
+    // w_t = gamma_bar_t * u_t; gamma_bar_t = (1/K) sum over the completions that reach t
+    double wmax = 0.0;
+    for (int t = tid; t < Tp; t += kDesignThreads) {
+      double acc = 0.0;
+      for (int j = 0; j < K; ++j)
+        if (t < L[p * K + j]) acc = __dadd_rn(acc, static_cast<double>(gamma[off[j] + t]));
+      double v = __ddiv_rn(acc, static_cast<double>(K));
+      if (u) v = __dmul_rn(v, static_cast<double>(u[static_cast<int64_t>(p) * T_max + t]));
+      w[t] = v;
+      wmax = fmax(wmax, v);
+    }
+#pragma unroll
+    for (int o = 16; o >= 1; o >>= 1) wmax = fmax(wmax, __shfl_xor_sync(0xffffffffu, wmax, o));
+    if (lane == 0) red_d[wid] = wmax;
+    __syncthreads();
+    double wm = 0.0;
+    for (int i = 0; i < kDesignThreads / 32; ++i) wm = fmax(wm, red_d[i]);
+    const double fl = __dmul_rn(1e-12, wm);
+    for (int t = tid; t < Tp; t += kDesignThreads) w[t] = wm > 0.0 ? (w[t] > fl ? w[t] : fl) : 1.0;
+    __syncthreads();
+    if (tid == 0) {
+      double* bW = ws.bW + static_cast<int64_t>(p) * T_max;
+      int32_t* bn = ws.bn + static_cast<int64_t>(p) * T_max;
+      if (strategy == PS_DESIGN_OPTIMIZED) {
+        // the smallest saturated prefix s whose suffix design starts at or below 1
+        int s = 0;
+        for (; s < Tp; ++s) {
+          monotone_design_dev(w + s, Tp - s, __dsub_rn(Bp, static_cast<double>(s)), xi + s, bW, bn);
+          if (xi[s] <= 1.0) break;
+        }
+        for (int t = 0; t < s && t < Tp; ++t) xi[t] = 1.0;
+      } else {
+        double tot = 0.0;
+        for (int t = 0; t < Tp; ++t) tot = __dadd_rn(tot, __dsqrt_rn(w[t]));
+        for (int t = 0; t < Tp; ++t) xi[t] = __ddiv_rn(__dmul_rn(Bp, __dsqrt_rn(w[t])), tot);
+        for (int t = 1; t < Tp; ++t) xi[t] = fmin(xi[t - 1], xi[t]);
+        for (int t = 0; t < Tp; ++t) xi[t] = fmin(xi[t], 1.0);
+      }
+    }
+  } else if (strategy == PS_DESIGN_UNIFORM) {
+    for (int t = tid; t < Tp; t += kDesignThreads)
+      xi[t] = __ddiv_rn(static_cast<double>(Tp - t), static_cast<double>(Tp));
+  } else if (strategy == PS_DESIGN_FIXED) {
+    for (int t = tid; t < Tp; t += kDesignThreads) xi[t] = (t + 1 <= param) ? 1.0 : 0.0;
+  } else {  // PS_DESIGN_TIME_PRIOR: xi_t = exp(-lam t), sum_t xi_t = budget, lam by bisection
+    auto budget_at = [&](double lam) {
+      double part = 0.0;
+      for (int t = tid; t < Tp; t += kDesignThreads) part += exp(-lam * t);
+#pragma unroll
+      for (int o = 16; o >= 1; o >>= 1) part += __shfl_xor_sync(0xffffffffu, part, o);
+      __syncthreads();
+      if (lane == 0) red_d[wid] = part;
+      __syncthreads();
+      double tot = 0.0;
+      for (int i = 0; i < kDesignThreads / 32; ++i) tot += red_d[i];
+      return tot;
+    };
+    if (static_cast<double>(Tp) <= Bp) {
+      if (tid == 0) lam_s = 0.0;
+    } else {
+      double lo = 0.0, hi = 1.0;
+      for (int it = 0; it < 64 && budget_at(hi) > Bp; ++it) hi *= 2.0;
+      for (int it = 0; it < 200; ++it) {
+        const double mid = 0.5 * (lo + hi);
+        if (budget_at(mid) > Bp) lo = mid;
+        else hi = mid;
+      }
+      if (tid == 0) lam_s = hi;
+    }
+    __syncthreads();
+    for (int t = tid; t < Tp; t += kDesignThreads) xi[t] = exp(-lam_s * t);
+  }
+  __syncthreads();
+
+  // masses q_h = floor((xi_h - xi_{h+1}) 2^62); excess over 2^62 comes off the largest mass
+  uint64_t* qp = q + static_cast<int64_t>(p) * T_max;
+  unsigned long long sum = 0, best = 0;
+  int besti = INT_MAX;
+  for (int t = tid; t < T_max; t += kDesignThreads) {
+    uint64_t v = 0;
+    if (t < Tp) {
+      const double d = __dsub_rn(xi[t], t + 1 < Tp ? xi[t + 1] : 0.0);
+      v = d > 0.0 ? __double2ull_rz(floor(__dmul_rn(d, 4611686018427387904.0))) : 0ull;
+    }
+    qp[t] = v;
+    if (xi_out) xi_out[static_cast<int64_t>(p) * T_max + t] = t < Tp ? xi[t] : 0.0;
+    sum += v;
+    if (v > best || (v == best && t < besti)) {
+      best = v;
+      besti = t;
+    }
+  }
+#pragma unroll
+  for (int o = 16; o >= 1; o >>= 1) {
+    sum += __shfl_xor_sync(0xffffffffu, sum, o);
+    const unsigned long long ob = __shfl_xor_sync(0xffffffffu, best, o);
+    const int oi = __shfl_xor_sync(0xffffffffu, besti, o);
+    if (ob > best || (ob == best && oi < besti)) {
+      best = ob;
+      besti = oi;
+    }
+  }
+  __syncthreads();
+  if (lane == 0) {
+    red_u[wid] = sum;
+    red_b[wid] = best;
+    red_i[wid] = besti;
+  }
+  __syncthreads();
+  if (tid == 0) {
+    unsigned long long s = 0, b = 0;
+    int bi = INT_MAX;
+    for (int i = 0; i < kDesignThreads / 32; ++i) {
+      s += red_u[i];
+      const unsigned long long v = red_b[i];
+      if (v > b || (v == b && red_i[i] < bi)) {
+        b = v;
+        bi = red_i[i];
+      }
+    }
+    if (s > kOne62 && bi < T_max) qp[bi] -= (s - kOne62);
+  }
+}
+
+}  // namespace psk
+
+using namespace psk;
+
+extern "C" {
+
+// Score-proxy workspace: header | ztok [N] f32 | hn [N] f32 | part [S][N] float4 (S as many as fit,
+// up to one per 256-column vocabulary tile).
+static size_t proxy_fixed(int64_t N) { return kWsHeader + al256(sizeof(float) * N) * 2; }
+
+size_t ps_lmhead_score_proxy_workspace_size(int64_t N, int d, int V, int dtype) {
+  if (N < 0 || V < 1 || d < 8 || dtype != PS_DTYPE_BF16) return 0;
+  return proxy_fixed(N) + sizeof(float4) * static_cast<size_t>(fwd_tile_splits_bf16(V)) * N;
+}
+
+int ps_lmhead_score_proxy(int64_t N, int d, int V, int dtype, const void* Hrows, const void* W, const int32_t* tok,
+                          float* gamma, float* logp, void* ws, size_t ws_bytes, ps_stream_t stream) {
+  if (N < 0 || N > INT32_MAX || V < 1 || d < 8 || d % 8) return PS_ERR_INVALID_ARG;
+  if (dtype != PS_DTYPE_BF16) return PS_ERR_UNSUPPORTED;
+  if (N > 0 && (!Hrows || !W || !tok || !gamma)) return PS_ERR_INVALID_ARG;
+  if (N > 0 && ((reinterpret_cast<uintptr_t>(Hrows) & 15) || (reinterpret_cast<uintptr_t>(W) & 15)))
+    return PS_ERR_INVALID_ARG;
+  if (!device_is_sm103()) return PS_ERR_UNSUPPORTED;
+  if (ws == nullptr || (reinterpret_cast<uintptr_t>(ws) & 255)) return PS_ERR_WORKSPACE;
+  const size_t fixed = proxy_fixed(N);
+  int S = fwd_tile_splits_bf16(V);
+  if (N > 0) {
+    const size_t room = ws_bytes > fixed ? ws_bytes - fixed : 0;
+    const size_t fit = room / (sizeof(float4) * static_cast<size_t>(N));
+    if (fit < static_cast<size_t>(S)) S = static_cast<int>(fit);
+    if (S < 1) return PS_ERR_WORKSPACE;
+  }
+  if (ws_bytes < fixed) return PS_ERR_WORKSPACE;
+  cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
+  if (cudaMemsetAsync(ws, 0, kWsHeader, s) != cudaSuccess) return PS_ERR_CUDA;
+  if (N == 0) return PS_OK;
+  uint8_t* base = static_cast<uint8_t*>(ws);
+  float* ztok = reinterpret_cast<float*>(base + kWsHeader);
+  float* hn = reinterpret_cast<float*>(base + kWsHeader + al256(sizeof(float) * N));
+  float4* part = reinterpret_cast<float4*>(base + fixed);
+  uint32_t* status = static_cast<uint32_t*>(ws);
+  row_sqnorm_kernel<<<num_sms_current() * 8, 256, 0, s>>>(N, d, 1, Hrows, hn);
+  if (cudaGetLastError() != cudaSuccess) return PS_ERR_CUDA;
+  const int splits = choose_fwd_splits_bf16(N, d, V, num_sms_current(), S);
+  int rc = proxy_gemm_bf16(N, d, V, Hrows, W, tok, part, ztok, splits, status, s);
+  if (rc != PS_OK) return rc;
+  proxy_finalize_kernel<<<static_cast<unsigned>((N + 255) / 256), 256, 0, s>>>(N, V, splits, part, ztok, hn, tok,
+                                                                                gamma, logp, status);
+  return cudaGetLastError() == cudaSuccess ? PS_OK : PS_ERR_CUDA;
+}
+
+static DesignWs design_ws(void* ws, int P, int K, int T_max) {
+  uint8_t* b = static_cast<uint8_t*>(ws) + kWsHeader;
+  const size_t pt = static_cast<size_t>(P) * T_max;
+  DesignWs d;
+  d.w = reinterpret_cast<double*>(b);
+  b += al256(sizeof(double) * pt);
+  d.xi = reinterpret_cast<double*>(b);
+  b += al256(sizeof(double) * pt);
+  d.bW = reinterpret_cast<double*>(b);
+  b += al256(sizeof(double) * pt);
+  d.bn = reinterpret_cast<int32_t*>(b);
+  b += al256(sizeof(int32_t) * pt);
+  d.off = reinterpret_cast<int64_t*>(b);
+  return d;
+}
+
+size_t ps_design_cutoffs_workspace_size(int P, int K, int T_max) {
+  if (P < 1 || K < 1 || T_max < 1) return 0;
+  const size_t pt = static_cast<size_t>(P) * T_max;
+  return kWsHeader + al256(sizeof(double) * pt) * 3 + al256(sizeof(int32_t) * pt) +
+         al256(sizeof(int64_t) * static_cast<size_t>(P) * K);
+}
+
+int ps_design_cutoffs(int P, int K, int T_max, const int32_t* L, const float* gamma_full, const float* u,
+                      double budget, int strategy, double param, uint64_t* q, double* xi, void* ws, size_t ws_bytes,
+                      ps_stream_t stream) {
+  if (P < 1 || K < 1 || T_max < 1 || T_max > (1 << 24) || !L || !q) return PS_ERR_INVALID_ARG;
+  if (static_cast<int64_t>(P) * K > INT32_MAX) return PS_ERR_INVALID_ARG;
+  if (strategy < PS_DESIGN_OPTIMIZED || strategy > PS_DESIGN_FIXED) return PS_ERR_INVALID_ARG;
+  const bool uses_gamma = strategy == PS_DESIGN_OPTIMIZED || strategy == PS_DESIGN_HEURISTIC;
+  if (uses_gamma && !gamma_full) return PS_ERR_INVALID_ARG;
+  if ((uses_gamma || strategy == PS_DESIGN_TIME_PRIOR) && !(budget > 0.0)) return PS_ERR_INVALID_ARG;
+  if (strategy == PS_DESIGN_FIXED && !(param >= 1.0)) return PS_ERR_INVALID_ARG;
+  if (ws == nullptr || (reinterpret_cast<uintptr_t>(ws) & 255) ||
+      ws_bytes < ps_design_cutoffs_workspace_size(P, K, T_max))
+    return PS_ERR_WORKSPACE;
+  cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
+  if (cudaMemsetAsync(ws, 0, kWsHeader, s) != cudaSuccess) return PS_ERR_CUDA;
+  design_kernel<<<P, kDesignThreads, 0, s>>>(K, T_max, L, gamma_full, u, budget, strategy, param, q, xi,
+                                              design_ws(ws, P, K, T_max), static_cast<uint32_t*>(ws));
+  return cudaGetLastError() == cudaSuccess ? PS_OK : PS_ERR_CUDA;
+}
+
+}  // extern "C"

@@ -20,6 +20,10 @@ int fwd_splits_f32(int V);
 int fwd_gemm_f32(int64_t N, int d, int V, const float* Hpk, const float* W, const int32_t* tok, float2* part,
                  float* ztok, uint32_t* status, cudaStream_t s);
 
+// Score-proxy GEMM (the forward's schedule): part [splits][N] (max2, s1, s2, 0), ztok [N].
+int proxy_gemm_bf16(int64_t N, int d, int V, const void* Hrows, const void* W, const int32_t* tok, float4* part,
+                    float* ztok, int splits, uint32_t* status, cudaStream_t s);
+
 // Backward for one chunk of rows [0, rc) of already offset pointers: recompute dZ into
 // dz ([rc][ldz], operand dtype), then dH = dZ W and dW (+)= dZ^T Hpk.
 int bwd_chunk_bf16(int64_t rc, int d, int V, const void* Hpk, const void* W, const int32_t* tok,

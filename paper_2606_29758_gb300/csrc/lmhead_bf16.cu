@@ -70,6 +70,72 @@ struct FwdLseEpi {
   }
 };
 
+// Score proxy of the cutoff design (Appendix D): besides the running max m (log2 units, over all
+// columns) keep r1 = sum_{v != o} 2^(x_v - m) and r2 = sum_{v != o} 4^(x_v - m) -- the two
+// logsumexp reductions of ||p||^2 = exp(LSE(2z) - 2 LSE(z)) with the chosen column o left out, so
+// that ||e_o - p||^2 = (r1^2 + r2) / (e_o + r1)^2 keeps its relative accuracy when p(o) -> 1
+// (1 - 2 p(o) + ||p||^2 would cancel there).
+struct FwdProxyEpi {
+  struct Params {
+    const int32_t* tok;
+    int M, N;
+    float4* part;   // [splits][M] (m2, s1, s2, 0)
+    float* ztok;
+  };
+  struct State {
+    float m2, s1, s2;
+    int tok;
+  };
+  static __device__ __forceinline__ void begin_unit(const Params& p, State& st, int row, int) {
+    st.m2 = -INFINITY;
+    st.s1 = 0.f;
+    st.s2 = 0.f;
+    st.tok = row < p.M ? __ldg(p.tok + row) : -1;
+  }
+  static __device__ __forceinline__ void chunk(const Params& p, State& st, int row, int col0,
+                                               const uint32_t (&r)[32]) {
+    if (col0 >= p.N) return;
+    float x[32];
+    const int nv = p.N - col0;
+#pragma unroll
+    for (int j = 0; j < 32; ++j) x[j] = (j < nv) ? __uint_as_float(r[j]) * kLog2e : -INFINITY;
+    float c0 = fmaxf(x[0], x[1]), c1 = fmaxf(x[2], x[3]);
+#pragma unroll
+    for (int j = 4; j < 32; j += 4) {
+      c0 = fmaxf(c0, fmaxf(x[j], x[j + 1]));
+      c1 = fmaxf(c1, fmaxf(x[j + 2], x[j + 3]));
+    }
+    const float mn = fmaxf(st.m2, fmaxf(c0, c1));
+    const int rel = st.tok - col0;
+    if (static_cast<unsigned>(rel) < 32u) {
+      float zt = 0.f;
+#pragma unroll
+      for (int j = 0; j < 32; ++j)
+        if (j == rel) {
+          zt = __uint_as_float(r[j]);
+          x[j] = -INFINITY;   // the chosen column stays out of r1 and r2
+        }
+      p.ztok[row] = zt;
+    }
+    float a0 = 0.f, a1 = 0.f, b0 = 0.f, b1 = 0.f;
+#pragma unroll
+    for (int j = 0; j < 32; j += 2) {
+      const float e0 = exp2f(x[j] - mn), e1 = exp2f(x[j + 1] - mn);
+      a0 += e0;
+      a1 += e1;
+      b0 = fmaf(e0, e0, b0);
+      b1 = fmaf(e1, e1, b1);
+    }
+    const float f = exp2f(st.m2 - mn);
+    st.s1 = st.s1 * f + (a0 + a1);
+    st.s2 = st.s2 * (f * f) + (b0 + b1);
+    st.m2 = mn;
+  }
+  static __device__ __forceinline__ void end_unit(const Params& p, State& st, int row, int split) {
+    if (row < p.M) p.part[static_cast<size_t>(split) * p.M + row] = make_float4(st.m2, st.s1, st.s2, 0.f);
+  }
+};
+
 struct BwdDzEpi {
   struct Params {
     const int32_t* tok;
@@ -356,6 +422,17 @@ int fwd_gemm_bf16(int64_t N, int d, int V, const void* Hpk, const void* W, const
 // large operand) is read from DRAM once and the small operand once per wave.
 constexpr int kBandRecompute = 48;
 constexpr int kBandGrad = 1;
+
+int proxy_gemm_bf16(int64_t N, int d, int V, const void* Hrows, const void* W, const int32_t* tok, float4* part,
+                    float* ztok, int splits, uint32_t* status, cudaStream_t s) {
+  CUtensorMap ta, tb;
+  if (!map_kmajor(&ta, Hrows, N, d, d, kBM * kFwdHalves) || !map_kmajor(&tb, W, V, d, d, kBRowsBox))
+    return PS_ERR_INVALID_ARG;
+  FwdProxyEpi::Params ep{tok, static_cast<int>(N), V, part, ztok};
+  const int workers = num_sms_current();
+  const int band = splits == fwd_tile_splits_bf16(V) ? fwd_band_max(d) : (workers + splits - 1) / splits;
+  return launch_gemm_single<false, false, FwdProxyEpi, kFwdHalves>(ta, tb, N, V, d, splits, band, ep, status, s);
+}
 
 int bwd_chunk_bf16(int64_t rc, int d, int V, const void* Hpk, const void* W, const int32_t* tok,
                    const float* lse, const float* coef, float* dH, float* dW, int dw_accumulate, void* dz,

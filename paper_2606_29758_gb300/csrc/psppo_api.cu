@@ -80,7 +80,7 @@ __global__ void __launch_bounds__(kSampThreads)
                           int32_t* __restrict__ n, float* __restrict__ w_tab, uint32_t* status) {
   extern __shared__ uint64_t xs[];  // [K] draws
   __shared__ uint64_t warp_tot[32];
-  __shared__ uint64_t carry_s;
+  __shared__ uint64_t carry_s, total_s;
   const int p = blockIdx.x;
   const int tid = threadIdx.x;
   const int64_t wrow = static_cast<int64_t>(p) * T_max;
@@ -104,10 +104,30 @@ __global__ void __launch_bounds__(kSampThreads)
     for (int t = tid; t < T_max; t += blockDim.x) w_tab[wrow + t] = 1.0f;
     return;
   }
+  const int lane = tid & 31, wid = tid >> 5;
+  // Total mass U[T] (saturating). Exact mode requires 2^62; in the H = 0 mode the deficit
+  // 2^62 - U[T] is Pr(H = 0) and the survival is S[t] = U[T] - U[t-1].
+  {
+    uint64_t part = 0;
+    for (int t = tid; t < T_max; t += blockDim.x) {
+      const uint64_t m = q[wrow + t];
+      part = sat_add(part, m > kOne62 ? kSatCap : m);
+    }
+#pragma unroll
+    for (int o = 16; o >= 1; o >>= 1) part = sat_add(part, __shfl_xor_sync(0xffffffffu, part, o));
+    if (lane == 0) warp_tot[wid] = part;
+    __syncthreads();
+    if (tid == 0) {
+      uint64_t tot = 0;
+      for (int w = 0; w < kSampThreads / 32; ++w) tot = sat_add(tot, warp_tot[w]);
+      total_s = tot;
+      if (tot > kOne62 || (mode == PS_MODE_TRUNC && tot != kOne62)) raise_status(status, PS_DEV_BAD_PMF);
+    }
+  }
   if (tid == 0) carry_s = 0;
   __syncthreads();
+  const uint64_t total = total_s > kOne62 ? kOne62 : total_s;
 
-  const int lane = tid & 31, wid = tid >> 5;
   for (int base = 0; base < T_max; base += kSampThreads) {
     const int t = base + tid;  // 0-based: bucket h = t + 1
     uint64_t m = t < T_max ? q[wrow + t] : 0ull;
@@ -138,13 +158,13 @@ __global__ void __launch_bounds__(kSampThreads)
     const uint64_t incl = sat_add(carry, sat_add(before, v));  // U[h]
     const uint64_t excl = sat_add(carry, sat_add(before, v - m > kSatCap ? kSatCap : v - m));
     if (t < T_max) {
-      // S[t+1] = 2^62 - U[t]; weight 2^62 / S (f64 divide, rounded once to f32)
+      // S[t+1] = U[T] - U[t]; weight 2^62 / S (f64 divide, rounded once to f32)
       float wt;
-      if (excl >= kOne62) {
+      if (excl >= total) {
         wt = INFINITY;
         if (excl > kOne62) raise_status(status, PS_DEV_BAD_PMF);
       } else {
-        const double S = __ull2double_rn(kOne62 - excl);
+        const double S = __ull2double_rn(total - excl);
         wt = __double2float_rn(__ddiv_rn(4611686018427387904.0, S));
       }
       w_tab[wrow + t] = wt;
@@ -163,7 +183,7 @@ __global__ void __launch_bounds__(kSampThreads)
     if (tid == kSampThreads - 1) carry_s = incl;
     __syncthreads();
   }
-  if (tid == 0 && carry_s != kOne62) raise_status(status, PS_DEV_BAD_PMF);
+  // (the total was checked before the scan; a draw at or above U[T] leaves H = n = 0)
 }
 
 // ================================================================== K2: packing
@@ -473,8 +493,8 @@ int ps_sample_cutoffs(int P, int K, int T_max, const uint64_t* q, const int32_t*
                       ps_stream_t stream) {
   if (P < 1 || K < 1 || K > 8192 || T_max < 1 || T_max > (1 << 24) || traj_base < 0) return PS_ERR_INVALID_ARG;
   if (static_cast<int64_t>(P) * K > INT32_MAX) return PS_ERR_INVALID_ARG;
-  if (mode != PS_MODE_TRUNC && mode != PS_MODE_FULL) return PS_ERR_INVALID_ARG;
-  if ((mode == PS_MODE_TRUNC && q == nullptr) || !L || !H || !n || !w_tab) return PS_ERR_INVALID_ARG;
+  if (mode != PS_MODE_TRUNC && mode != PS_MODE_FULL && mode != PS_MODE_TRUNC_ZERO) return PS_ERR_INVALID_ARG;
+  if ((mode != PS_MODE_FULL && q == nullptr) || !L || !H || !n || !w_tab) return PS_ERR_INVALID_ARG;
   cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
   int rc = begin_call(ws, ws_bytes, ps_sample_cutoffs_workspace_size(P, K, T_max), s);
   if (rc != PS_OK) return rc;

@@ -222,3 +222,18 @@ def to_device(b: Batch, device: str) -> Dict[str, object]:
         "oldlogp_full": torch.from_numpy(b.oldlogp_full).to(device),
     }
     return d
+
+
+_S_GAMMA, _S_UNC = 7, 8
+
+
+def draw_design_inputs(cfg: Config, L: np.ndarray):
+    """Inputs of the cutoff-design step: a positive per-token score gamma in completion order
+    (a decaying trend times lognormal noise, so that adjacent timesteps often violate the
+    monotone order) and a reward-uncertainty proxy u [P, T_max] on [0.02, 0.25]."""
+    g = _rng(cfg.seed, _S_GAMMA)
+    total = int(L.sum())
+    t = np.concatenate([np.arange(int(n), dtype=np.float64) for n in L])
+    gamma = (cfg.d * (1.0 + 3.0 * np.exp(-t / 200.0)) * np.exp(0.7 * g.standard_normal(total))).astype(np.float32)
+    u = _rng(cfg.seed, _S_UNC).uniform(0.02, 0.25, size=(cfg.P, int(L.max()))).astype(np.float32)
+    return gamma, u
