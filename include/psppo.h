@@ -198,12 +198,34 @@ int ps_lmhead_ppo_bwd(int64_t N, int d, int V, int dtype, const void* Hpk, const
  * gamma [N] f32 and, if logp is not NULL, log p_i(o_i) [N] f32.
  * Hrows [N][d] bf16, W [V][d] bf16 (bf16 only: other dtypes return PS_ERR_UNSUPPORTED),
  * tok [N] int32 (PS_DEV_BAD_TOKEN and NaN outputs for ids outside [0, V)).
- * Workspace: like the forward, as many vocabulary partials (16 B per row each) as fit, up
- * to ps_lmhead_score_proxy_workspace_size(); at least one per row.
+ * topk (0..16): if > 0, the same pass also returns each row's topk most likely next tokens,
+ * top_idx [N][topk] int32 (descending probability, lower id first on ties) and their
+ * probabilities top_prob [N][topk] f32 -- the input of ps_reward_uncertainty (Appendix I
+ * uses 16).
+ * Workspace: as many vocabulary partials per row as fit (16 B each; with topk > 0, 144 B each
+ * and at most 16), up to ps_lmhead_score_proxy_workspace_size(); at least one per row.
  * ------------------------------------------------------------------------- */
-size_t ps_lmhead_score_proxy_workspace_size(int64_t N, int d, int V, int dtype);
+size_t ps_lmhead_score_proxy_workspace_size(int64_t N, int d, int V, int dtype, int topk);
 int ps_lmhead_score_proxy(int64_t N, int d, int V, int dtype, const void* Hrows, const void* W,
                           const int32_t* tok, float* gamma, float* logp,
+                          int topk, int32_t* top_idx, float* top_prob,
+                          void* ws, size_t ws_bytes, ps_stream_t stream);
+
+/* ---------------------------------------------------------------------------
+ * ps_reward_uncertainty -- the reward-uncertainty proxy u_t of each prompt and step.
+ *
+ * Appendix E (Eq. ut_def): u_t = 1/2 - 1/2 || p pi_G(.|t) - (1 - p) pi_B(.|t) ||_1, an upper
+ * bound on E[Var(R | S_t) | x] for binary rewards, estimated from the group's K completions:
+ * p = fraction with R >= 0.5; pi_G / pi_B average the old-policy next-token distributions at
+ * step t over the successful / unsuccessful completions that reach t (an empty class adds 0).
+ * Each distribution is its top-k tokens plus one "other" symbol with its remaining mass
+ * (the top-k approximation of Appendix I). Output u [P][T_max] f32, 0 beyond a group's
+ * horizon. Inputs: L [B], R [B] f32, top_idx [sum L][topk] int32 and top_prob [sum L][topk]
+ * f32 in completion order (as from ps_lmhead_score_proxy). Limits: K <= 64, 1 <= topk <= 16.
+ * ------------------------------------------------------------------------- */
+size_t ps_reward_uncertainty_workspace_size(int P, int K);
+int ps_reward_uncertainty(int P, int K, int T_max, const int32_t* L, const float* R, int topk,
+                          const int32_t* top_idx, const float* top_prob, float* u,
                           void* ws, size_t ws_bytes, ps_stream_t stream);
 
 /* ---------------------------------------------------------------------------

@@ -238,3 +238,67 @@ def design_cutoff_masses(L, K, gamma_full, u, B, strategy, param=0.0):
         q[p, :Tp] = masses_from_xi(xi)
         xi_all[p, :Tp] = xi
     return q, xi_all
+
+
+# ----------------------------------------------------------------------------- reward uncertainty
+def topk_policy(H, W, k):
+    """Per row, the k most likely next tokens of softmax(W h) and their probabilities (float64;
+    ties go to the lower token id). Appendix I: the u_t estimate keeps the top k = 16."""
+    H = np.asarray(H, dtype=np.float64)
+    W = np.asarray(W, dtype=np.float64)
+    idx = np.empty((H.shape[0], k), dtype=np.int64)
+    prob = np.empty((H.shape[0], k))
+    for r0 in range(0, H.shape[0], 128):
+        z = H[r0:r0 + 128] @ W.T
+        m = z.max(axis=1, keepdims=True)
+        p = np.exp(z - m)
+        p /= p.sum(axis=1, keepdims=True)
+        order = np.lexsort((np.broadcast_to(np.arange(z.shape[1]), z.shape), -z), axis=1)[:, :k]
+        idx[r0:r0 + 128] = order
+        prob[r0:r0 + 128] = np.take_along_axis(p, order, axis=1)
+    return idx, prob
+
+
+def reward_uncertainty(L, K, R, top_idx, top_prob):
+    """u[p][t-1] = 1/2 - 1/2 || p_hat pi_G(.|t) - (1 - p_hat) pi_B(.|t) ||_1 (Appendix E, Eq. ut_def),
+    estimated from the group's K completions (Appendix E, last paragraph):
+
+    p_hat = fraction of the group with R = 1 (R >= 0.5 counts as success); pi_G(.|t) / pi_B(.|t)
+    average the old-policy next-token distributions at step t over the successful / unsuccessful
+    completions that reach t (a class with none contributes 0). Each distribution is represented by
+    its top-k tokens plus one "other" symbol holding its remaining mass (the top-k approximation of
+    Appendix I; with k = V it is the definition). Rows of top_idx / top_prob are in completion order.
+    Steps beyond the group's horizon get u = 0.
+    """
+    L = np.asarray(L)
+    Bn = len(L)
+    P = Bn // K
+    T_max = int(L.max())
+    off = np.concatenate([[0], np.cumsum(L)])
+    u = np.zeros((P, T_max))
+    for p in range(P):
+        ks = list(range(p * K, (p + 1) * K))
+        succ = [k for k in ks if float(R[k]) >= 0.5]
+        fail = [k for k in ks if float(R[k]) < 0.5]
+        p_hat = len(succ) / K
+        Tp = int(max(L[k] for k in ks))
+        for t in range(Tp):
+            g_alive = [k for k in succ if L[k] > t]
+            b_alive = [k for k in fail if L[k] > t]
+            coef = {}
+            for k in g_alive:
+                coef[k] = p_hat / len(g_alive)
+            for k in b_alive:
+                coef[k] = -(1.0 - p_hat) / len(b_alive)
+            mass = {}
+            other = 0.0
+            for k, c in coef.items():
+                row = off[k] + t
+                tot = 0.0
+                for v, pv in zip(top_idx[row], top_prob[row]):
+                    mass[int(v)] = mass.get(int(v), 0.0) + c * float(pv)
+                    tot += float(pv)
+                other += c * (1.0 - tot)
+            l1 = sum(abs(x) for x in mass.values()) + abs(other)
+            u[p, t] = min(0.5, max(0.0, 0.5 - 0.5 * l1))
+    return u

@@ -31,6 +31,7 @@ EXPORTS = [
     "ps_diag_gemm_bf16", "ps_diag_wait_timeout", "ps_lmhead_ppo_fwd_noalloc",
     "ps_lmhead_score_proxy_workspace_size", "ps_lmhead_score_proxy",
     "ps_design_cutoffs_workspace_size", "ps_design_cutoffs",
+    "ps_reward_uncertainty_workspace_size", "ps_reward_uncertainty",
 ]
 PS_DESIGN_OPTIMIZED, PS_DESIGN_HEURISTIC, PS_DESIGN_UNIFORM, PS_DESIGN_TIME_PRIOR, PS_DESIGN_FIXED = range(5)
 
@@ -75,8 +76,11 @@ _SIGS = {
     "ps_diag_gemm_bf16": (_i32, [_i32, _i32, _i32, _i32, _i32, _vp, _i64, _vp, _i64, _vp, _i64, _i32, _i32, _vp, _sz,
                                  _vp]),
     "ps_diag_wait_timeout": (_i32, [_u64, _vp, _sz, _vp]),
-    "ps_lmhead_score_proxy_workspace_size": (_sz, [_i64, _i32, _i32, _i32]),
-    "ps_lmhead_score_proxy": (_i32, [_i64, _i32, _i32, _i32, _vp, _vp, _vp, _vp, _vp, _vp, _sz, _vp]),
+    "ps_lmhead_score_proxy_workspace_size": (_sz, [_i64, _i32, _i32, _i32, _i32]),
+    "ps_lmhead_score_proxy": (_i32, [_i64, _i32, _i32, _i32, _vp, _vp, _vp, _vp, _vp, _i32, _vp, _vp, _vp, _sz,
+                                     _vp]),
+    "ps_reward_uncertainty_workspace_size": (_sz, [_i32, _i32]),
+    "ps_reward_uncertainty": (_i32, [_i32, _i32, _i32, _vp, _vp, _i32, _vp, _vp, _vp, _vp, _sz, _vp]),
     "ps_design_cutoffs_workspace_size": (_sz, [_i32, _i32, _i32]),
     "ps_design_cutoffs": (_i32, [_i32, _i32, _i32, _vp, _vp, _vp, _f64, _i32, _f64, _vp, _vp, _vp, _sz, _vp]),
     "ps_lmhead_ppo_fwd_noalloc": (_i32, [_i64, _i32, _i32, _i32, _vp, _vp, _vp, _vp, _vp, _vp, _f64, _f64,
@@ -200,14 +204,25 @@ def ps_lmhead_ppo_fwd_noalloc(N, d, V, dtype, Hpk, W, tok, oldlogp, adv, w, eps,
     _check(rc, "ps_lmhead_ppo_fwd_noalloc")
 
 
-def ps_lmhead_score_proxy_workspace_size(N: int, d: int, V: int, dtype: int) -> int:
-    return lib().ps_lmhead_score_proxy_workspace_size(N, d, V, dtype)
+def ps_lmhead_score_proxy_workspace_size(N: int, d: int, V: int, dtype: int, topk: int = 0) -> int:
+    return lib().ps_lmhead_score_proxy_workspace_size(N, d, V, dtype, topk)
 
 
-def ps_lmhead_score_proxy(N, d, V, dtype, Hrows, W, tok, gamma, logp, ws, stream=None):
-    rc = lib().ps_lmhead_score_proxy(N, d, V, dtype, _ptr(Hrows), _ptr(W), _ptr(tok), _ptr(gamma), _ptr(logp),
-                                     _ptr(ws), _nbytes(ws), _stream(stream))
+def ps_lmhead_score_proxy(N, d, V, dtype, Hrows, W, tok, gamma, logp, ws, topk=0, top_idx=None, top_prob=None,
+                          stream=None):
+    rc = lib().ps_lmhead_score_proxy(N, d, V, dtype, _ptr(Hrows), _ptr(W), _ptr(tok), _ptr(gamma), _ptr(logp), topk,
+                                     _ptr(top_idx), _ptr(top_prob), _ptr(ws), _nbytes(ws), _stream(stream))
     _check(rc, "ps_lmhead_score_proxy")
+
+
+def ps_reward_uncertainty_workspace_size(P: int, K: int) -> int:
+    return lib().ps_reward_uncertainty_workspace_size(P, K)
+
+
+def ps_reward_uncertainty(P, K, T_max, L, R, topk, top_idx, top_prob, u, ws, stream=None):
+    rc = lib().ps_reward_uncertainty(P, K, T_max, _ptr(L), _ptr(R), topk, _ptr(top_idx), _ptr(top_prob), _ptr(u),
+                                     _ptr(ws), _nbytes(ws), _stream(stream))
+    _check(rc, "ps_reward_uncertainty")
 
 
 def ps_design_cutoffs_workspace_size(P: int, K: int, T_max: int) -> int:

@@ -57,7 +57,9 @@ __global__ void row_sqnorm_kernel(int64_t N, int d, int is_bf16, const void* __r
 __global__ void proxy_finalize_kernel(int64_t N, int V, int splits, const float4* __restrict__ part,
                                       const float* __restrict__ ztok, const float* __restrict__ hn,
                                       const int32_t* __restrict__ tok, float* __restrict__ gamma,
-                                      float* __restrict__ logp, uint32_t* status) {
+                                      float* __restrict__ logp, int topk_k, const float2* __restrict__ topk_part,
+                                      int32_t* __restrict__ top_idx, float* __restrict__ top_prob,
+                                      uint32_t* status) {
   const int64_t i = static_cast<int64_t>(blockIdx.x) * blockDim.x + threadIdx.x;
   if (i >= N) return;
   float m = -INFINITY;
@@ -82,6 +84,126 @@ __global__ void proxy_finalize_kernel(int64_t N, int V, int splits, const float4
   const double tot = eo + S1;
   gamma[i] = static_cast<float>(static_cast<double>(hn[i]) * ((S1 * S1 + S2) / (tot * tot)));
   if (logp) logp[i] = static_cast<float>((x - log2(tot)) * 0.6931471805599453);
+  if (topk_k > 0) {
+    // merge the ranges' lists (each descending, lower column first on ties), ranges in order
+    float v[16];
+    int id[16];
+#pragma unroll
+    for (int j = 0; j < 16; ++j) {
+      v[j] = -INFINITY;
+      id[j] = -1;
+    }
+    for (int sp = 0; sp < splits; ++sp) {
+      const float2* lst = topk_part + (static_cast<int64_t>(sp) * N + i) * 16;
+      for (int c = 0; c < 16; ++c) {
+        const float2 e = lst[c];
+        float xv = e.x;
+        int xi = __float_as_int(e.y);
+        if (!(xv > v[15])) continue;
+#pragma unroll
+        for (int j = 0; j < 16; ++j) {
+          const bool take = xv > v[j];
+          const float tv = v[j];
+          const int ti = id[j];
+          v[j] = take ? xv : tv;
+          id[j] = take ? xi : ti;
+          xv = take ? tv : xv;
+          xi = take ? ti : xi;
+        }
+      }
+    }
+#pragma unroll
+    for (int j = 0; j < 16; ++j) {
+      if (j < topk_k) {
+        top_idx[i * topk_k + j] = id[j];
+        top_prob[i * topk_k + j] =
+            static_cast<float>(exp2(static_cast<double>(v[j]) * 1.4426950408889634 - m) / tot);
+      }
+    }
+  }
+}
+
+// ================================================================== reward uncertainty
+// One warp per (prompt, step t): the group's completions that reach t contribute their top-k
+// next-token probabilities with coefficient p_hat / |G_t| (success) or -(1 - p_hat) / |B_t|
+// (failure); u_t = 1/2 - 1/2 (sum over distinct tokens |sum of contributions| + |other mass|).
+constexpr int kUncWarps = 4;
+__global__ void __launch_bounds__(kUncWarps * 32)
+    uncertainty_kernel(int P, int K, int T_max, const int32_t* __restrict__ L, const float* __restrict__ R,
+                       int topk, const int32_t* __restrict__ top_idx, const float* __restrict__ top_prob,
+                       const int64_t* __restrict__ off, float* __restrict__ u) {
+  extern __shared__ uint8_t smem[];
+  const int lane = threadIdx.x & 31, wid = threadIdx.x >> 5;
+  const int cap = K * topk;
+  int32_t* etok = reinterpret_cast<int32_t*>(smem) + wid * cap;
+  double* eval = reinterpret_cast<double*>(smem + sizeof(int32_t) * kUncWarps * cap + 16) + wid * cap;
+  const int64_t task = static_cast<int64_t>(blockIdx.x) * kUncWarps + wid;
+  if (task >= static_cast<int64_t>(P) * T_max) return;
+  const int p = static_cast<int>(task / T_max);
+  const int t = static_cast<int>(task % T_max);   // 0-based step
+  int nG = 0, gA = 0, bA = 0, Tp = 0;
+  for (int j = 0; j < K; ++j) {
+    const int k = p * K + j;
+    const bool g = R[k] >= 0.5f;
+    nG += g;
+    gA += (g && L[k] > t);
+    bA += (!g && L[k] > t);
+    Tp = max(Tp, L[k]);
+  }
+  if (t >= Tp) {
+    if (lane == 0) u[static_cast<int64_t>(p) * T_max + t] = 0.f;
+    return;
+  }
+  const double phat = static_cast<double>(nG) / K;
+  const double cg = gA > 0 ? phat / gA : 0.0, cb = bA > 0 ? -(1.0 - phat) / bA : 0.0;
+  // entries of the alive completions, in completion order
+  int E = 0;
+  double other = 0.0;
+  for (int j = 0; j < K; ++j) {
+    const int k = p * K + j;
+    if (L[k] <= t) continue;
+    const double c = R[k] >= 0.5f ? cg : cb;
+    const int64_t row = off[k] + t;
+    double tot = 0.0;
+    for (int i = lane; i < topk; i += 32) {
+      etok[E + i] = top_idx[row * topk + i];
+      const double pv = top_prob[row * topk + i];
+      eval[E + i] = c * pv;
+      tot += pv;
+    }
+#pragma unroll
+    for (int o = 16; o >= 1; o >>= 1) tot += __shfl_xor_sync(0xffffffffu, tot, o);
+    other += c * (1.0 - tot);
+    E += topk;
+  }
+  __syncwarp();
+  double acc = 0.0;
+  for (int e = lane; e < E; e += 32) {
+    const int tk = etok[e];
+    bool first = true;
+    for (int f = 0; f < e && first; ++f) first = etok[f] != tk;
+    if (!first) continue;
+    double sum = 0.0;
+    for (int f = e; f < E; ++f)
+      if (etok[f] == tk) sum += eval[f];
+    acc += fabs(sum);
+  }
+#pragma unroll
+  for (int o = 16; o >= 1; o >>= 1) acc += __shfl_xor_sync(0xffffffffu, acc, o);
+  if (lane == 0) {
+    const double l1 = acc + fabs(other);
+    u[static_cast<int64_t>(p) * T_max + t] = static_cast<float>(fmin(0.5, fmax(0.0, 0.5 - 0.5 * l1)));
+  }
+}
+
+__global__ void group_offsets_kernel(int B, const int32_t* __restrict__ L, int64_t* __restrict__ off) {
+  if (threadIdx.x == 0 && blockIdx.x == 0) {
+    int64_t o = 0;
+    for (int k = 0; k < B; ++k) {
+      off[k] = o;
+      o += L[k];
+    }
+  }
 }
 
 // ================================================================== design
@@ -297,28 +419,38 @@ using namespace psk;
 extern "C" {
 
 // Score-proxy workspace: header | ztok [N] f32 | hn [N] f32 | part [S][N] float4 (S as many as fit,
-// up to one per 256-column vocabulary tile).
+// up to one per 256-column vocabulary tile) -- with top-k: part [S][N] float4 and topk [S][N][16]
+// float2 for S <= 16 contiguous vocabulary ranges.
 static size_t proxy_fixed(int64_t N) { return kWsHeader + al256(sizeof(float) * N) * 2; }
+static size_t proxy_per_split(int64_t N, int topk) {
+  return (sizeof(float4) + (topk > 0 ? sizeof(float2) * 16 : 0)) * static_cast<size_t>(N);
+}
+static int proxy_max_splits(int V, int topk) { return topk > 0 ? 16 : fwd_tile_splits_bf16(V); }
 
-size_t ps_lmhead_score_proxy_workspace_size(int64_t N, int d, int V, int dtype) {
-  if (N < 0 || V < 1 || d < 8 || dtype != PS_DTYPE_BF16) return 0;
-  return proxy_fixed(N) + sizeof(float4) * static_cast<size_t>(fwd_tile_splits_bf16(V)) * N;
+size_t ps_lmhead_score_proxy_workspace_size(int64_t N, int d, int V, int dtype, int topk) {
+  if (N < 0 || V < 1 || d < 8 || dtype != PS_DTYPE_BF16 || topk < 0 || topk > 16) return 0;
+  int S = proxy_max_splits(V, topk);
+  if (S > fwd_tile_splits_bf16(V)) S = fwd_tile_splits_bf16(V);
+  return proxy_fixed(N) + proxy_per_split(N, topk) * S;
 }
 
 int ps_lmhead_score_proxy(int64_t N, int d, int V, int dtype, const void* Hrows, const void* W, const int32_t* tok,
-                          float* gamma, float* logp, void* ws, size_t ws_bytes, ps_stream_t stream) {
-  if (N < 0 || N > INT32_MAX || V < 1 || d < 8 || d % 8) return PS_ERR_INVALID_ARG;
+                          float* gamma, float* logp, int topk, int32_t* top_idx, float* top_prob, void* ws,
+                          size_t ws_bytes, ps_stream_t stream) {
+  if (N < 0 || N > INT32_MAX || V < 1 || d < 8 || d % 8 || topk < 0 || topk > 16) return PS_ERR_INVALID_ARG;
   if (dtype != PS_DTYPE_BF16) return PS_ERR_UNSUPPORTED;
   if (N > 0 && (!Hrows || !W || !tok || !gamma)) return PS_ERR_INVALID_ARG;
+  if (N > 0 && topk > 0 && (!top_idx || !top_prob)) return PS_ERR_INVALID_ARG;
   if (N > 0 && ((reinterpret_cast<uintptr_t>(Hrows) & 15) || (reinterpret_cast<uintptr_t>(W) & 15)))
     return PS_ERR_INVALID_ARG;
   if (!device_is_sm103()) return PS_ERR_UNSUPPORTED;
   if (ws == nullptr || (reinterpret_cast<uintptr_t>(ws) & 255)) return PS_ERR_WORKSPACE;
   const size_t fixed = proxy_fixed(N);
-  int S = fwd_tile_splits_bf16(V);
+  int S = proxy_max_splits(V, topk);
+  if (S > fwd_tile_splits_bf16(V)) S = fwd_tile_splits_bf16(V);
   if (N > 0) {
     const size_t room = ws_bytes > fixed ? ws_bytes - fixed : 0;
-    const size_t fit = room / (sizeof(float4) * static_cast<size_t>(N));
+    const size_t fit = room / proxy_per_split(N, topk);
     if (fit < static_cast<size_t>(S)) S = static_cast<int>(fit);
     if (S < 1) return PS_ERR_WORKSPACE;
   }
@@ -330,14 +462,44 @@ int ps_lmhead_score_proxy(int64_t N, int d, int V, int dtype, const void* Hrows,
   float* ztok = reinterpret_cast<float*>(base + kWsHeader);
   float* hn = reinterpret_cast<float*>(base + kWsHeader + al256(sizeof(float) * N));
   float4* part = reinterpret_cast<float4*>(base + fixed);
+  float2* tpart = reinterpret_cast<float2*>(base + fixed + sizeof(float4) * static_cast<size_t>(S) * N);
   uint32_t* status = static_cast<uint32_t*>(ws);
   row_sqnorm_kernel<<<num_sms_current() * 8, 256, 0, s>>>(N, d, 1, Hrows, hn);
   if (cudaGetLastError() != cudaSuccess) return PS_ERR_CUDA;
   const int splits = choose_fwd_splits_bf16(N, d, V, num_sms_current(), S);
-  int rc = proxy_gemm_bf16(N, d, V, Hrows, W, tok, part, ztok, splits, status, s);
+  int rc = topk > 0 ? proxy_topk_gemm_bf16(N, d, V, Hrows, W, tok, part, tpart, ztok, splits, status, s)
+                    : proxy_gemm_bf16(N, d, V, Hrows, W, tok, part, ztok, splits, status, s);
   if (rc != PS_OK) return rc;
-  proxy_finalize_kernel<<<static_cast<unsigned>((N + 255) / 256), 256, 0, s>>>(N, V, splits, part, ztok, hn, tok,
-                                                                                gamma, logp, status);
+  proxy_finalize_kernel<<<static_cast<unsigned>((N + 127) / 128), 128, 0, s>>>(
+      N, V, splits, part, ztok, hn, tok, gamma, logp, topk, tpart, top_idx, top_prob, status);
+  return cudaGetLastError() == cudaSuccess ? PS_OK : PS_ERR_CUDA;
+}
+
+size_t ps_reward_uncertainty_workspace_size(int P, int K) {
+  if (P < 1 || K < 1) return 0;
+  return kWsHeader + al256(sizeof(int64_t) * static_cast<size_t>(P) * K);
+}
+
+int ps_reward_uncertainty(int P, int K, int T_max, const int32_t* L, const float* R, int topk,
+                          const int32_t* top_idx, const float* top_prob, float* u, void* ws, size_t ws_bytes,
+                          ps_stream_t stream) {
+  if (P < 1 || K < 1 || K > 64 || T_max < 1 || topk < 1 || topk > 16) return PS_ERR_INVALID_ARG;
+  if (!L || !R || !top_idx || !top_prob || !u) return PS_ERR_INVALID_ARG;
+  if (ws == nullptr || (reinterpret_cast<uintptr_t>(ws) & 255) ||
+      ws_bytes < ps_reward_uncertainty_workspace_size(P, K))
+    return PS_ERR_WORKSPACE;
+  cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
+  if (cudaMemsetAsync(ws, 0, kWsHeader, s) != cudaSuccess) return PS_ERR_CUDA;
+  int64_t* off = reinterpret_cast<int64_t*>(static_cast<uint8_t*>(ws) + kWsHeader);
+  group_offsets_kernel<<<1, 32, 0, s>>>(P * K, L, off);
+  if (cudaGetLastError() != cudaSuccess) return PS_ERR_CUDA;
+  const size_t smem = (sizeof(int32_t) + sizeof(double)) * kUncWarps * K * topk + 16;
+  if (cudaFuncSetAttribute(uncertainty_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                           static_cast<int>(smem)) != cudaSuccess)
+    return PS_ERR_CUDA;
+  const int64_t tasks = static_cast<int64_t>(P) * T_max;
+  uncertainty_kernel<<<static_cast<unsigned>((tasks + kUncWarps - 1) / kUncWarps), kUncWarps * 32, smem, s>>>(
+      P, K, T_max, L, R, topk, top_idx, top_prob, off, u);
   return cudaGetLastError() == cudaSuccess ? PS_OK : PS_ERR_CUDA;
 }
 

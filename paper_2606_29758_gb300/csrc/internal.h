@@ -24,6 +24,12 @@ int fwd_gemm_f32(int64_t N, int d, int V, const float* Hpk, const float* W, cons
 int proxy_gemm_bf16(int64_t N, int d, int V, const void* Hrows, const void* W, const int32_t* tok, float4* part,
                     float* ztok, int splits, uint32_t* status, cudaStream_t s);
 
+// Score proxy plus the 16 largest logits per row and vocabulary range (contiguous ranges, at most
+// 16): topk [splits][N][16] (logit, column bits).
+int proxy_topk_gemm_bf16(int64_t N, int d, int V, const void* Hrows, const void* W, const int32_t* tok,
+                         float4* part, float2* topk, float* ztok, int splits, uint32_t* status, cudaStream_t s);
+// The forward's chooser with at most max_splits contiguous vocabulary ranges (exported for the proxy).
+
 // Backward for one chunk of rows [0, rc) of already offset pointers: recompute dZ into
 // dz ([rc][ldz], operand dtype), then dH = dZ W and dW (+)= dZ^T Hpk.
 int bwd_chunk_bf16(int64_t rc, int d, int V, const void* Hpk, const void* W, const int32_t* tok,

@@ -136,6 +136,73 @@ struct FwdProxyEpi {
   }
 };
 
+// FwdProxyEpi plus the 16 largest logits of the unit's vocabulary range (Appendix I: u_t uses
+// the top 16 next tokens). The list stays sorted (descending, lower column first on ties) in
+// registers; a 32-column slice is scanned only if its maximum beats the current 16th value.
+constexpr int kTopK = 16;
+struct FwdProxyTopkEpi {
+  struct Params {
+    const int32_t* tok;
+    int M, N;
+    float4* part;     // [splits][M] (m2, r1, r2, 0)
+    float2* topk;     // [splits][M][16] (logit, column as float bits)
+    float* ztok;
+  };
+  struct State {
+    FwdProxyEpi::State base;
+    float v[kTopK];
+    int id[kTopK];
+  };
+  static __device__ __forceinline__ void begin_unit(const Params& p, State& st, int row, int split) {
+    FwdProxyEpi::Params bp{p.tok, p.M, p.N, p.part, p.ztok};
+    FwdProxyEpi::begin_unit(bp, st.base, row, split);
+#pragma unroll
+    for (int j = 0; j < kTopK; ++j) {
+      st.v[j] = -INFINITY;
+      st.id[j] = -1;
+    }
+  }
+  static __device__ __forceinline__ void chunk(const Params& p, State& st, int row, int col0,
+                                               const uint32_t (&r)[32]) {
+    if (col0 >= p.N) return;
+    const int nv = p.N - col0;
+    float cm = -INFINITY;
+#pragma unroll
+    for (int j = 0; j < 32; ++j)
+      if (j < nv) cm = fmaxf(cm, __uint_as_float(r[j]));
+    if (cm > st.v[kTopK - 1]) {
+#pragma unroll
+      for (int j = 0; j < 32; ++j) {
+        float x = j < nv ? __uint_as_float(r[j]) : -INFINITY;
+        if (x > st.v[kTopK - 1]) {
+          int c = col0 + j;
+#pragma unroll
+          for (int i = 0; i < kTopK; ++i) {
+            const bool take = x > st.v[i];
+            const float tv = st.v[i];
+            const int ti = st.id[i];
+            st.v[i] = take ? x : tv;
+            st.id[i] = take ? c : ti;
+            x = take ? tv : x;
+            c = take ? ti : c;
+          }
+        }
+      }
+    }
+    FwdProxyEpi::Params bp{p.tok, p.M, p.N, p.part, p.ztok};
+    FwdProxyEpi::chunk(bp, st.base, row, col0, r);
+  }
+  static __device__ __forceinline__ void end_unit(const Params& p, State& st, int row, int split) {
+    FwdProxyEpi::Params bp{p.tok, p.M, p.N, p.part, p.ztok};
+    FwdProxyEpi::end_unit(bp, st.base, row, split);
+    if (row < p.M) {
+      float2* dst = p.topk + (static_cast<size_t>(split) * p.M + row) * kTopK;
+#pragma unroll
+      for (int j = 0; j < kTopK; ++j) dst[j] = make_float2(st.v[j], __int_as_float(st.id[j]));
+    }
+  }
+};
+
 struct BwdDzEpi {
   struct Params {
     const int32_t* tok;
@@ -432,6 +499,16 @@ int proxy_gemm_bf16(int64_t N, int d, int V, const void* Hrows, const void* W, c
   const int workers = num_sms_current();
   const int band = splits == fwd_tile_splits_bf16(V) ? fwd_band_max(d) : (workers + splits - 1) / splits;
   return launch_gemm_single<false, false, FwdProxyEpi, kFwdHalves>(ta, tb, N, V, d, splits, band, ep, status, s);
+}
+
+int proxy_topk_gemm_bf16(int64_t N, int d, int V, const void* Hrows, const void* W, const int32_t* tok,
+                         float4* part, float2* topk, float* ztok, int splits, uint32_t* status, cudaStream_t s) {
+  CUtensorMap ta, tb;
+  if (!map_kmajor(&ta, Hrows, N, d, d, kBM) || !map_kmajor(&tb, W, V, d, d, kBRowsBox)) return PS_ERR_INVALID_ARG;
+  FwdProxyTopkEpi::Params ep{tok, static_cast<int>(N), V, part, topk, ztok};
+  const int workers = num_sms_current();
+  const int band = (workers + splits - 1) / splits;
+  return launch_gemm_single<false, false, FwdProxyTopkEpi, 1>(ta, tb, N, V, d, splits, band, ep, status, s);
 }
 
 int bwd_chunk_bf16(int64_t rc, int d, int V, const void* Hpk, const void* W, const int32_t* tok,

@@ -135,3 +135,103 @@ def test_score_proxy_matches_oracle(name, w_scale):
     if w_scale > 1.0:
         assert sel.sum() > 10
         np.testing.assert_allclose(g[sel] / hn[sel], part_ref[sel], rtol=2e-4, atol=2e-5)
+
+
+@pytest.mark.parametrize("name,w_scale", [("mid", 12.0), ("head7b_small", 4.0)])
+def test_proxy_top16_matches_oracle(name, w_scale):
+    from paper_2606_29758_gb300 import _binding as B
+    cfg = get_config(name, w_std=0.02 * w_scale)
+    b = make_batch(cfg, device="cuda")
+    hid, W = widen(cfg, b.hid_full), widen(cfg, b.W)
+    N, k = len(b.tok_full), 16
+    gamma = torch.empty(N, device="cuda")
+    tidx = torch.empty(N, k, dtype=torch.int32, device="cuda")
+    tprob = torch.empty(N, k, device="cuda")
+    ws = torch.empty(B.ps_lmhead_score_proxy_workspace_size(N, cfg.d, cfg.V, B.PS_DTYPE_BF16, k), dtype=torch.uint8,
+                     device="cuda")
+    B.ps_lmhead_score_proxy(N, cfg.d, cfg.V, B.PS_DTYPE_BF16, b.dev["hid_full"], b.dev["W"], b.dev["tok_full"], gamma,
+                            None, ws, k, tidx, tprob)
+    torch.cuda.synchronize()
+    assert B.ps_workspace_status(ws)[0] == B.PS_OK
+    g_ref, _ = design.score_proxy(hid, W, b.tok_full)
+    np.testing.assert_allclose(gamma.cpu().numpy(), g_ref, rtol=2e-4)
+    ridx, rprob = design.topk_policy(hid, W, k)
+    gi, gp = tidx.cpu().numpy(), tprob.cpu().numpy()
+    z = hid @ W.T
+    m = z.max(axis=1, keepdims=True)
+    P = np.exp(z - m)
+    P /= P.sum(axis=1, keepdims=True)
+    rows = np.arange(N)[:, None]
+    # the GPU's probabilities are those of its tokens, descending
+    np.testing.assert_allclose(gp, P[rows, gi], rtol=2e-4, atol=1e-9)
+    assert np.all(np.diff(gp, axis=1) <= 1e-7)
+    # its set is a top-k set: same mass as the oracle's, and the same tokens away from near-ties
+    np.testing.assert_allclose(P[rows, gi].sum(axis=1), rprob.sum(axis=1), rtol=1e-5)
+    zk = np.sort(z, axis=1)[:, ::-1]
+    clear = (zk[:, k - 1] - zk[:, k]) > 1e-3
+    assert np.array_equal(np.sort(gi[clear], axis=1), np.sort(ridx[clear], axis=1))
+
+
+@pytest.mark.parametrize("name", ["mid", "7b"])
+def test_reward_uncertainty_matches_oracle(name):
+    from paper_2606_29758_gb300 import _binding as B
+    cfg = get_config(name)
+    L = draw_lengths(cfg)
+    N, k = int(L.sum()), 16
+    rng = np.random.default_rng(2)
+    # seeded top-16 lists over a small shared vocabulary so that completions overlap
+    idx = np.stack([rng.choice(64, size=k, replace=False) for _ in range(N)]).astype(np.int32)
+    prob = rng.dirichlet(np.ones(k + 1), size=N)[:, :k].astype(np.float32)
+    R = (rng.random(cfg.B) < 0.5).astype(np.float32)
+    R[:cfg.K] = 1.0                                   # one all-success group (u = 0 where all alive)
+    T = int(L.max())
+    u = torch.empty(cfg.P, T, device="cuda")
+    ws = torch.empty(B.ps_reward_uncertainty_workspace_size(cfg.P, cfg.K), dtype=torch.uint8, device="cuda")
+    B.ps_reward_uncertainty(cfg.P, cfg.K, T, torch.from_numpy(L).cuda(), torch.from_numpy(R).cuda(), k,
+                            torch.from_numpy(idx).cuda(), torch.from_numpy(prob).cuda(), u, ws)
+    torch.cuda.synchronize()
+    assert B.ps_workspace_status(ws)[0] == B.PS_OK
+    ref = design.reward_uncertainty(L, cfg.K, R, idx, prob)
+    np.testing.assert_allclose(u.cpu().numpy(), ref, atol=2e-7)
+
+
+def test_design_then_update_end_to_end():
+    # proxy + top-16 -> u -> optimized design -> H = 0 sampling -> packing -> forward -> backward,
+    # all on the device; every status clear and the outputs finite
+    from paper_2606_29758_gb300 import _binding as B
+    from paper_2606_29758_gb300 import PassShape, UpdatePass
+    cfg = get_config("mid")
+    b = make_batch(cfg, device="cuda")
+    D = b.dev
+    N, T, k = b.total_len, b.T_max, 16
+    gamma = torch.empty(N, device="cuda")
+    tidx = torch.empty(N, k, dtype=torch.int32, device="cuda")
+    tprob = torch.empty(N, k, device="cuda")
+    ws_p = torch.empty(B.ps_lmhead_score_proxy_workspace_size(N, cfg.d, cfg.V, B.PS_DTYPE_BF16, k),
+                       dtype=torch.uint8, device="cuda")
+    B.ps_lmhead_score_proxy(N, cfg.d, cfg.V, B.PS_DTYPE_BF16, D["hid_full"], D["W"], D["tok_full"], gamma, None,
+                            ws_p, k, tidx, tprob)
+    u = torch.empty(cfg.P, T, device="cuda")
+    ws_u = torch.empty(B.ps_reward_uncertainty_workspace_size(cfg.P, cfg.K), dtype=torch.uint8, device="cuda")
+    B.ps_reward_uncertainty(cfg.P, cfg.K, T, D["L"], D["R"], k, tidx, tprob, u, ws_u)
+    q = torch.empty(cfg.P, T, dtype=torch.int64, device="cuda")
+    xi = torch.empty(cfg.P, T, dtype=torch.float64, device="cuda")
+    ws_d = torch.empty(B.ps_design_cutoffs_workspace_size(cfg.P, cfg.K, T), dtype=torch.uint8, device="cuda")
+    B.ps_design_cutoffs(cfg.P, cfg.K, T, D["L"], gamma, u, 40.0, B.PS_DESIGN_OPTIMIZED, 0.0, q, xi, ws_d)
+    up = UpdatePass(PassShape(cfg.P, cfg.K, T, cfg.d, cfg.V, N), eps=cfg.eps, loss_scale=cfg.loss_scale,
+                    mode=B.PS_MODE_TRUNC_ZERO)
+    up.run(q, D["L"], D["R"], D["tok_full"], D["oldlogp_full"], D["hid_full"], D["W"], 3, 0)
+    torch.cuda.synchronize()
+    for ws in (ws_p, ws_u, ws_d):
+        assert B.ps_workspace_status(ws)[0] == B.PS_OK
+    up.check_status()
+    uu = u.cpu().numpy()
+    assert np.all((uu >= 0) & (uu <= 0.5))
+    x = xi.cpu().numpy()
+    for p in range(cfg.P):
+        Tp = int(b.L[p * cfg.K:(p + 1) * cfg.K].max())
+        assert x[p, :Tp].sum() == pytest.approx(min(40.0, Tp), rel=1e-12)
+    Nr = up.N
+    assert torch.isfinite(up.loss).all() and torch.isfinite(up.dH[:Nr]).all() and torch.isfinite(up.dW).all()
+    # weights are 1/xi of the realised distribution
+    assert float(up.w[:Nr].min()) >= 1.0

@@ -151,3 +151,62 @@ def test_score_proxy_is_the_squared_head_gradient_norm():
                 g[v, c] = (lp(Wp) - lp(Wn)) / (2 * eps)
         assert gamma[i] == pytest.approx(float((g * g).sum()), rel=1e-7)
         assert logp[i] == pytest.approx(lp(W), rel=1e-13)
+
+
+def _u_full(L, K, R, P_rows):
+    """Eq. ut_def with the full next-token distributions (no top-k)."""
+    V = P_rows.shape[1]
+    idx = np.tile(np.arange(V), (P_rows.shape[0], 1))
+    return design.reward_uncertainty(L, K, R, idx, P_rows)
+
+
+def test_uncertainty_closed_cases():
+    L = np.array([3, 3, 3, 3])
+    V = 4
+    one = np.zeros((12, V))
+    one[:, 1] = 1.0
+    # every completion succeeds: the reward is certain, u = 0
+    assert np.all(_u_full(L, 4, np.ones(4), one) == 0.0)
+    # half succeed but all predict the same distribution: nothing separates them, u = 1/2
+    assert np.allclose(_u_full(L, 4, np.array([1, 1, 0, 0]), one), 0.5)
+    # successes put their mass on token 0, failures on token 3: the prefix decides the reward, u = 0
+    sep = np.zeros((12, V))
+    sep[0:6, 0] = 1.0
+    sep[6:12, 3] = 1.0
+    assert np.allclose(_u_full(L, 4, np.array([1, 1, 0, 0]), sep), 0.0)
+    # Bernoulli bound: u <= 1/2 always, and min(p_hat, 1 - p_hat) <= ... >= 0
+    rng = np.random.default_rng(0)
+    Pr = rng.dirichlet(np.ones(V), size=12)
+    u = _u_full(L, 4, np.array([1, 0, 0, 0]), Pr)
+    assert np.all((u >= 0) & (u <= 0.5))
+
+
+def test_topk_route_with_every_token_is_the_definition():
+    rng = np.random.default_rng(5)
+    K, V = 4, 12
+    L = rng.integers(2, 7, size=2 * K)
+    R = np.array([1, 0, 1, 1, 0, 0, 1, 0], dtype=np.float32)
+    H = rng.standard_normal((int(L.sum()), 3))
+    W = rng.standard_normal((V, 3)) * 1.3
+    idx_full, p_full = design.topk_policy(H, W, V)
+    u_full = design.reward_uncertainty(L, K, R, idx_full, p_full)
+    # with k = V the top-k route equals the definition written with full distributions
+    z = H @ W.T
+    Pr = np.exp(z - z.max(axis=1, keepdims=True))
+    Pr /= Pr.sum(axis=1, keepdims=True)
+    np.testing.assert_allclose(u_full, _u_full(L, K, R, Pr), atol=1e-14)
+    # dropping only tokens of zero probability changes nothing
+    Pr2 = np.concatenate([Pr, np.zeros((Pr.shape[0], 5))], axis=1)
+    np.testing.assert_allclose(_u_full(L, K, R, Pr2), u_full, atol=1e-14)
+    # and u stays within [0, 1/2] for every k
+    for k in (1, 3, 6):
+        idx, pk = design.topk_policy(H, W, k)
+        uk = design.reward_uncertainty(L, K, R, idx, pk)
+        assert np.all((uk >= 0) & (uk <= 0.5))
+
+
+def test_topk_policy_orders_and_ties():
+    W = np.array([[1.0], [3.0], [3.0], [0.5]])
+    idx, p = design.topk_policy(np.array([[1.0]]), W, 3)
+    assert list(idx[0]) == [1, 2, 0]
+    assert p[0, 0] == pytest.approx(p[0, 1]) and p[0].sum() < 1.0
