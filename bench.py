@@ -36,9 +36,10 @@ WORKLOAD = "7b"
 MEASURED_PEAKS = os.path.join(ROOT, "MEASURED_PEAKS.json")
 FALLBACK_PEAKS = {"hbm_gbs": 6800.0, "bf16_tflops": 1900.0, "bf16_tflops_sustained": 1700.0}
 
-# dram bytes (read + write) per launch of the forward GEMM, from the ncu capture named
-# below, scaled to this workload's rows; None until measured for the current kernel.
-FWD_GEMM_TRAFFIC = None
+# DRAM bytes (read + write) per launch of the forward GEMM on the 7b workload, the mean of the
+# eight launches in profiles/lmhead_pass_7b_launch_list.md (76.67 GB read + 0.92 GB written).
+# Reset to None whenever the forward kernel or its schedule changes.
+FWD_GEMM_TRAFFIC = {"7b": 77.59e9}
 
 
 def describe(cfg) -> str:
@@ -259,7 +260,7 @@ def run_ours(args):
                         "bwd": float(per[:, 2].mean())},
         "roofline": {"kernel": "umma_gemm_kernel<K,K,FwdLseEpi> (fused forward; + O(N) finalize)",
                      "bound": "tensor", "achieved": achieved_tf, "peak": peak_tf, "unit": "TFLOP/s",
-                     "frac": achieved_tf / peak_tf, "traffic": FWD_GEMM_TRAFFIC,
+                     "frac": achieved_tf / peak_tf, "traffic": FWD_GEMM_TRAFFIC.get(cfg.name),
                      "algorithmic_per_launch": f"2*N*d*V = {fwd_flops:.4g} FLOP",
                      "peak_note": f"bf16_tflops_sustained ({src}); kernel timed inside the step"},
         "e2e": {"value": e_rows / (e_ms * 1e-3), "unit": "tokens/s", "h2d_bytes_per_step": h2d,
