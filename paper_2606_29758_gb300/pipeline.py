@@ -104,3 +104,45 @@ class UpdatePass:
             rc, bits = B.ps_workspace_status(ws)
             if rc != B.PS_OK:
                 raise B.PsppoError(rc, f"{name} (device bits {bits:#x})")
+
+
+class InputStager:
+    """Double-buffered host -> device staging of the unpacked batch inputs.
+
+    Holds `slots` device copies of a dict of tensors (the per-batch inputs of UpdatePass.sample and
+    UpdatePass.pack) and a copy stream. `stage(host)` enqueues the host -> device copies of one batch
+    (pinned host tensors, so the copies are asynchronous) into the next slot and returns the slot;
+    `acquire(slot, stream)` makes `stream` wait for that slot's copies and returns its tensors;
+    `release(slot, stream)` marks the slot free once the work enqueued on `stream` so far is done, and
+    a later `stage` into the slot waits for that. Staging batch i + 1 before running the pass on
+    batch i lets the copy engine move the next batch while the tensor cores work on this one.
+    """
+
+    def __init__(self, like: dict, device: str = "cuda", slots: int = 2):
+        if slots < 1:
+            raise ValueError("slots must be >= 1")
+        self.bufs = [{k: torch.empty(v.shape, dtype=v.dtype, device=device) for k, v in like.items()}
+                     for _ in range(slots)]
+        self.copy_stream = torch.cuda.Stream(device=device)
+        self.ready = [torch.cuda.Event() for _ in range(slots)]
+        self.free = [torch.cuda.Event() for _ in range(slots)]
+        self.nbytes = sum(v.numel() * v.element_size() for v in like.values())
+        self._next = 0
+
+    def stage(self, host: dict) -> int:
+        j = self._next
+        self._next = (j + 1) % len(self.bufs)
+        dst = self.bufs[j]
+        with torch.cuda.stream(self.copy_stream):
+            self.copy_stream.wait_event(self.free[j])     # no-op until the slot has been released once
+            for k, t in host.items():
+                dst[k].copy_(t, non_blocking=True)
+            self.ready[j].record(self.copy_stream)
+        return j
+
+    def acquire(self, j: int, stream=None) -> dict:
+        (stream or torch.cuda.current_stream()).wait_event(self.ready[j])
+        return self.bufs[j]
+
+    def release(self, j: int, stream=None):
+        self.free[j].record(stream or torch.cuda.current_stream())

@@ -96,3 +96,39 @@ def test_forward_with_fewer_vocabulary_partials(name):
                             cfg.eps, cfg.loss_scale, loss, outs["lse"], outs["logp"], outs["ratio"], outs["coef"],
                             None, tiny_ws)
     assert e.value.status == B.PS_ERR_WORKSPACE
+
+
+def test_input_stager_overlapped_copies_give_the_resident_results():
+    # Two batches of one shape, copied from pinned host memory through the double-buffered stager
+    # while the previous pass runs, must give bit for bit the results of passes on resident inputs.
+    import torch
+    from paper_2606_29758_gb300 import InputStager
+    cfg = get_config("mid")
+    b = make_batch(cfg, device="cuda")
+    keys = ("q", "L", "R", "tok_full", "oldlogp_full", "hid_full")
+    A = {k: b.dev[k] for k in keys}
+    Bt = dict(A, R=1.0 - A["R"], tok_full=(A["tok_full"] + 7) % cfg.V, oldlogp_full=A["oldlogp_full"] - 0.01,
+              hid_full=A["hid_full"].flip(0).contiguous())
+    batches = [A, Bt, A, Bt, Bt]
+    ref = []
+    for i, X in enumerate(batches):
+        _, up = gpu_pass(cfg, b)           # allocate a pass of this shape, then rerun on X
+        up.run(X["q"], X["L"], X["R"], X["tok_full"], X["oldlogp_full"], X["hid_full"], b.dev["W"], cfg.seed, i)
+        torch.cuda.synchronize()
+        ref.append((up.N, up.loss.clone(), up.dH[:up.N].clone(), up.dW.clone()))
+    hosts = [{k: v.cpu().pin_memory() for k, v in X.items()} for X in batches]
+    _, up = gpu_pass(cfg, b)
+    stager = InputStager(hosts[0], device="cuda")
+    stream = torch.cuda.current_stream()
+    j = stager.stage(hosts[0])
+    for i in range(len(batches)):
+        X = stager.acquire(j, stream)
+        nxt = stager.stage(hosts[i + 1]) if i + 1 < len(batches) else None
+        up.run(X["q"], X["L"], X["R"], X["tok_full"], X["oldlogp_full"], X["hid_full"], b.dev["W"], cfg.seed, i)
+        stager.release(j, stream)
+        torch.cuda.synchronize()
+        N, loss, dH, dW = ref[i]
+        assert up.N == N
+        assert torch.equal(up.loss, loss) and torch.equal(up.dH[:N], dH) and torch.equal(up.dW, dW), i
+        j = nxt
+    up.check_status()
