@@ -121,5 +121,6 @@ def check_head(cfg, b, g, pk, rows=None, grads=True, report=None):
             assert stats["dW"] < GRAD_MAXREL, stats
     if report is not None:
         report.update(stats)
+        report["oracle_rows"], report["oracle_lse"], report["oracle_coef"] = idx, f["lse"], f["coef"]
     return stats
 

@@ -6,7 +6,10 @@ evaluate one by one (random rows, the largest weights, and rows where the clip b
 lse, logp, ratio, coef, row loss and the dH row. For dW, which sums over every row,
 two properties that hold at any size are checked: sum_v dW[v, :] = 0 (the softmax score
 e_o - p sums to zero over the vocabulary) within the bound set by the bf16 rounding of
-dZ, and loss = sum of row losses.
+dZ, and loss = sum of row losses. Then dW itself: the backward runs again over all N rows
+of the oracle's packed batch with the oracle's lse and coef on the sampled rows and coef = 0
+on every other row (whose dZ row is then zero), so dW = sum over the sampled rows, which the
+oracle evaluates on every vocabulary row that a sampled row chose plus 512 random ones.
 """
 import numpy as np
 import pytest
@@ -14,7 +17,7 @@ import torch
 
 from synthetic import get_config, make_batch
 
-from gpu_util import check_head, oracle_prefix
+from gpu_util import GRAD_MAXREL, check_head, oracle_prefix
 
 pytestmark = pytest.mark.gpu
 
@@ -67,7 +70,8 @@ def test_full_size(name):
     sel = torch.from_numpy(rows).cuda()
     dH[rows] = up.dH[sel].cpu().numpy()
     g["dH"] = dH
-    stats = check_head(cfg, b, g, pk, rows=rows)
+    rep = {}
+    stats = check_head(cfg, b, g, pk, rows=rows, report=rep)
     print(name, N, len(rows), stats)
 
     # loss = sum of row losses (the row losses are checked above)
@@ -82,3 +86,33 @@ def test_full_size(name):
     ratio = (colsum.abs() / (1.5 * bound + 1e-6 * up.dW.abs().max().double())).max().item()
     assert ratio < 1.0, ratio
     assert torch.isfinite(up.dW).all() and torch.isfinite(up.dH[:N]).all()
+
+    # dW at full size: same N, chunking and kernels; only the sampled rows carry a coefficient
+    from oracle import lmhead
+    from oracle.pipeline import widen
+    from paper_2606_29758_gb300 import _binding as B
+    idx, lse_o, coef_o = rep["oracle_rows"], rep["oracle_lse"], rep["oracle_coef"]
+    lse32 = np.zeros(N, dtype=np.float32)
+    coef32 = np.zeros(N, dtype=np.float32)
+    lse32[idx], coef32[idx] = lse_o.astype(np.float32), coef_o.astype(np.float32)
+    hid_o = torch.from_numpy(pk["hid"].view(np.int16)).cuda().view(torch.bfloat16)
+    tok_o = torch.from_numpy(pk["tok"].astype(np.int32)).cuda()
+    dH2 = torch.empty(N, cfg.d, dtype=torch.float32, device="cuda")
+    dW2 = torch.empty(cfg.V, cfg.d, dtype=torch.float32, device="cuda")
+    up.ws_bwd.zero_()
+    B.ps_lmhead_ppo_bwd(N, cfg.d, cfg.V, up.dcode, hid_o, D["W"], tok_o, torch.from_numpy(lse32).cuda(),
+                        torch.from_numpy(coef32).cuda(), dH2, dW2, B.PS_DW_OVERWRITE, up.ws_bwd)
+    torch.cuda.synchronize()
+    up.check_status()
+    vocab = np.unique(np.concatenate([pk["tok"][idx], rng.choice(cfg.V, size=512, replace=False)]))
+    _, dW_ref = lmhead.backward(widen(cfg, pk["hid"][idx]), widen(cfg, b.W), pk["tok"][idx],
+                                lse32[idx].astype(np.float64), coef32[idx].astype(np.float64),
+                                dh_rows=[], dw_vocab=vocab)
+    got = dW2[torch.from_numpy(vocab).cuda()].double().cpu().numpy()
+    err = float(np.abs(got - dW_ref).max() / np.abs(dW_ref).max())
+    print(name, "dW over", len(idx), "rows,", len(vocab), "vocab rows: max-rel", err)
+    assert err < GRAD_MAXREL, err
+    # every other row's dZ is zero, so the unsampled rows of dH vanish
+    others = torch.ones(N, dtype=torch.bool, device="cuda")
+    others[torch.from_numpy(idx).cuda()] = False
+    assert float(dH2[others].abs().max().item()) == 0.0
