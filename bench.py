@@ -236,6 +236,29 @@ def run_ours(args):
     torch.cuda.synchronize()
     h2d_ms = c0.elapsed_time(c1)
 
+    # ---- control: the same batch with every completion kept whole (H = L, all weights 1), the
+    # untruncated update that prefix sampling replaces; timed apart from the headline.
+    from paper_2606_29758_gb300 import PS_MODE_FULL
+    mode0 = up.mode
+    up.mode = PS_MODE_FULL
+    for i in range(2):
+        step(3000 + i)
+    barrier()
+    f0 = torch.cuda.Event(enable_timing=True)
+    f1 = torch.cuda.Event(enable_timing=True)
+    f_steps = 3
+    f0.record(stream)
+    f_rows = sum(step(3100 + i) for i in range(f_steps))
+    f1.record(stream)
+    barrier()
+    up.mode = mode0
+    up.check_status()
+    f_ms = f0.elapsed_time(f1) / f_steps
+    full_control = {"ms_per_step": f_ms, "rows_per_step": f_rows / f_steps,
+                    "tokens_per_s": f_rows / (f_ms * f_steps * 1e-3),
+                    "step_time_ratio_full_over_prefix": f_ms / (ms / args.steps),
+                    "note": "same batch, every completion kept whole (H = L, weights 1); 3 timed steps"}
+
     design = time_design_stage(cfg, b, dev, stream) if not args.no_design else None
 
     peaks, src = _peaks()
@@ -281,6 +304,7 @@ def run_ours(args):
                 "d2h_bytes_per_step": 8, "ms_per_step": e_ms / args.steps,
                 "h2d_alone_ms": h2d_ms, "h2d_alone_gbs": h2d / (h2d_ms * 1e-3) / 1e9,
                 "overlap": "next batch copied on a second stream during the current pass (InputStager)"},
+        "full_control": full_control,
         "gpu_launches": launches_per_step * args.steps,
         "clocks": clk,
     }

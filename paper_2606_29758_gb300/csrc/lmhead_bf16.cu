@@ -162,31 +162,46 @@ struct FwdProxyTopkEpi {
       st.id[j] = -1;
     }
   }
+  // Value j of the slice, picked by a select tree on the bits of j (keeps r in registers).
+  static __device__ __forceinline__ float pick32(const uint32_t (&r)[32], int j) {
+    float a[16];
+#pragma unroll
+    for (int i = 0; i < 16; ++i) a[i] = __uint_as_float((j & 1) ? r[2 * i + 1] : r[2 * i]);
+#pragma unroll
+    for (int i = 0; i < 8; ++i) a[i] = (j & 2) ? a[2 * i + 1] : a[2 * i];
+#pragma unroll
+    for (int i = 0; i < 4; ++i) a[i] = (j & 4) ? a[2 * i + 1] : a[2 * i];
+#pragma unroll
+    for (int i = 0; i < 2; ++i) a[i] = (j & 8) ? a[2 * i + 1] : a[2 * i];
+    return (j & 16) ? a[1] : a[0];
+  }
   static __device__ __forceinline__ void chunk(const Params& p, State& st, int row, int col0,
                                                const uint32_t (&r)[32]) {
     if (col0 >= p.N) return;
     const int nv = p.N - col0;
-    float cm = -INFINITY;
+    // Mask of the slice's values above the current 16th largest; after the first slices of a
+    // range it is almost always empty. The candidates are then inserted one at a time by one
+    // compact loop (a fully unrolled insertion per column overflows the instruction cache).
+    const float tau = st.v[kTopK - 1];
+    uint32_t m = 0;
 #pragma unroll
-    for (int j = 0; j < 32; ++j)
-      if (j < nv) cm = fmaxf(cm, __uint_as_float(r[j]));
-    if (cm > st.v[kTopK - 1]) {
+    for (int j = 0; j < 32; ++j) m |= (j < nv && __uint_as_float(r[j]) > tau) ? (1u << j) : 0u;
+#pragma unroll 1
+    while (m != 0u) {
+      const int j = __ffs(m) - 1;
+      m &= m - 1u;
+      float x = pick32(r, j);
+      if (!(x > st.v[kTopK - 1])) continue;   // the threshold rose since the mask was taken
+      int c = col0 + j;
 #pragma unroll
-      for (int j = 0; j < 32; ++j) {
-        float x = j < nv ? __uint_as_float(r[j]) : -INFINITY;
-        if (x > st.v[kTopK - 1]) {
-          int c = col0 + j;
-#pragma unroll
-          for (int i = 0; i < kTopK; ++i) {
-            const bool take = x > st.v[i];
-            const float tv = st.v[i];
-            const int ti = st.id[i];
-            st.v[i] = take ? x : tv;
-            st.id[i] = take ? c : ti;
-            x = take ? tv : x;
-            c = take ? ti : c;
-          }
-        }
+      for (int i = 0; i < kTopK; ++i) {
+        const bool take = x > st.v[i];
+        const float tv = st.v[i];
+        const int ti = st.id[i];
+        st.v[i] = take ? x : tv;
+        st.id[i] = take ? c : ti;
+        x = take ? tv : x;
+        c = take ? ti : c;
       }
     }
     FwdProxyEpi::Params bp{p.tok, p.M, p.N, p.part, p.ztok};
@@ -506,8 +521,11 @@ int proxy_topk_gemm_bf16(int64_t N, int d, int V, const void* Hrows, const void*
   CUtensorMap ta, tb;
   if (!map_kmajor(&ta, Hrows, N, d, d, kBM) || !map_kmajor(&tb, W, V, d, d, kBRowsBox)) return PS_ERR_INVALID_ARG;
   FwdProxyTopkEpi::Params ep{tok, static_cast<int>(N), V, part, topk, ztok};
+  // Units are contiguous vocabulary ranges; a band of row blocks whose rows fill the forward's L2
+  // share walks them range by range, so W is read from DRAM about once per band.
   const int workers = num_sms_current();
-  const int band = (workers + splits - 1) / splits;
+  int band = static_cast<int>(kFwdBandL2Bytes / (static_cast<double>(kBM) * d * 2.0));
+  if (band < (workers + splits - 1) / splits) band = (workers + splits - 1) / splits;
   return launch_gemm_single<false, false, FwdProxyTopkEpi, 1>(ta, tb, N, V, d, splits, band, ep, status, s);
 }
 
