@@ -124,7 +124,7 @@ int ps_sample_cutoffs(int P, int K, int T_max, const uint64_t* q, const int32_t*
  * row_traj (k), row_pos (t, 1-based).
  * h_num_rows: HOST pointer; if not NULL the call synchronises the stream and
  * stores N there.
- * Limits: d % 8 == 0 (bf16) or d % 4 == 0 (f32); sum L < 2^31.
+ * Limits: d >= 8 and d % 8 == 0 (bf16) or d % 4 == 0 (f32); sum L < 2^31.
  * ------------------------------------------------------------------------- */
 size_t ps_pack_prefixes_workspace_size(int P, int K);
 int ps_pack_prefixes(int P, int K, int T_max, int d, int dtype,
@@ -158,8 +158,8 @@ int ps_pack_prefixes(int P, int K, int T_max, int d, int dtype,
  * partial per row; the forward then splits the vocabulary into as many ranges as fit
  * (more passes over W). f32 needs the full size. Too small: PS_ERR_WORKSPACE, nothing
  * launched.
- * Limits: N >= 0 (N = 0 writes loss = 0), 1 <= V < 2^31, d % 8 == 0 (bf16) or
- * d % 4 == 0 (f32); 16-byte aligned Hpk and W.
+ * Limits: N >= 0 (N = 0 writes loss = 0), 1 <= V < 2^31, d >= 8 and d % 8 == 0 (bf16)
+ * or d % 4 == 0 (f32); 16-byte aligned Hpk and W.
  * ------------------------------------------------------------------------- */
 size_t ps_lmhead_ppo_fwd_workspace_size(int64_t N, int d, int V, int dtype);
 int ps_lmhead_ppo_fwd(int64_t N, int d, int V, int dtype, const void* Hpk, const void* W,

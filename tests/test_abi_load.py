@@ -67,3 +67,35 @@ def test_bad_arguments_are_rejected_before_any_launch(lib):
     assert L.ps_pack_prefixes(1, 1, 1, 8, 7, None, None, None, 1, None, None, None, None, 0,
                               None, None, None, None, None, None, None, None, None,
                               ctypes.POINTER(ctypes.c_int64)(), None, 0, None) == 1
+
+
+def test_size_limits_and_design_arguments_are_rejected_on_the_host(lib):
+    # Every case fails argument checks that run before the first CUDA call (no GPU here).
+    import ctypes
+    L = lib
+    INV = 1
+    z = (None,) * 4
+    # sampler: group larger than 8192, horizon beyond 2^24, unknown mode
+    assert L.ps_sample_cutoffs(1, 8193, 10, *z[:2], 0, 0, 0, 0, None, None, None, None, 0, None) == INV
+    assert L.ps_sample_cutoffs(1, 8, (1 << 24) + 1, *z[:2], 0, 0, 0, 0, None, None, None, None, 0, None) == INV
+    assert L.ps_sample_cutoffs(1, 8, 10, *z[:2], 0, 0, 0, 7, None, None, None, None, 0, None) == INV
+    # head: more rows than int32, a bf16 hidden size that is not a multiple of 8, an empty vocabulary
+    fwd = lambda N, d, V, dt: L.ps_lmhead_ppo_fwd(N, d, V, dt, None, None, None, None, None, None, 0.2, 1.0,  # noqa: E731
+                                                  None, None, None, None, None, None, None, 0, None)
+    assert fwd(1 << 31, 128, 1024, 0) == INV
+    assert fwd(10, 100, 1024, 0) == INV
+    assert fwd(10, 4, 1024, 0) == INV and fwd(10, 4, 1024, 1) == INV     # d >= 8 for both dtypes
+    assert fwd(10, 128, 0, 0) == INV
+    assert fwd(10, 128, 1024, 5) == INV
+    assert L.ps_lmhead_ppo_bwd(10, 128, 1024, 0, None, None, None, None, None, None, None, 7, None, 0, None) == INV
+    assert L.ps_lmhead_ppo_fwd_noalloc(10, 128, 0, 0, None, None, None, None, None, None, 0.2, 1.0,
+                                       None, None, None, None, None, None, None) == INV
+    assert L.ps_lmhead_ppo_fwd_workspace_size(10, 128, 0, 0) == 0
+    # design stage: top-k beyond 16, groups beyond 64 for u_t, unknown strategy, a fixed prefix below 1
+    assert L.ps_lmhead_score_proxy(10, 128, 1024, 0, None, None, None, None, None, 17, None, None, None, 0,
+                                   None) == INV
+    assert L.ps_reward_uncertainty(1, 65, 10, None, None, 16, None, None, None, None, 0, None) == INV
+    fake = ctypes.c_void_p(1 << 20)     # never dereferenced: the checks fail first
+    assert L.ps_design_cutoffs(1, 8, 10, fake, None, None, 4.0, 9, 0.0, fake, None, None, 0, None) == INV
+    assert L.ps_design_cutoffs(1, 8, 10, fake, None, None, 4.0, 4, 0.5, fake, None, None, 0, None) == INV
+    assert L.ps_design_cutoffs(1, 8, 10, fake, None, None, 0.0, 3, 0.0, fake, None, None, 0, None) == INV
