@@ -176,9 +176,10 @@ int ps_lmhead_ppo_fwd(int64_t N, int d, int V, int dtype, const void* Hpk, const
  *   dH = dZ W            [N][d] f32 (overwritten),
  *   dW = dZ^T Hpk        [V][d] f32 (overwritten, or added to with PS_DW_ACCUMULATE).
  * The logits are recomputed tile by tile; dZ is held, in the operand dtype, only
- * for one chunk of rows at a time inside the workspace: the chunk is the largest
- * multiple of 128 rows that fits (ws_bytes), so a larger workspace means fewer
- * chunks. dH or dW may be NULL to skip that product.
+ * for one chunk of rows at a time inside the workspace: the rows are split into as
+ * few chunks as the workspace holds (ws_bytes), of equal size rounded up to a
+ * multiple of 128 rows, so a larger workspace means fewer chunks. dH or dW may be
+ * NULL to skip that product.
  * Limits as for the forward; ws_bytes >= ps_lmhead_ppo_bwd_workspace_size(N, d, V,
  * dtype, 128) (one chunk of 128 rows).
  * ------------------------------------------------------------------------- */

@@ -618,8 +618,12 @@ int ps_lmhead_ppo_bwd(int64_t N, int d, int V, int dtype, const void* Hpk, const
   const int64_t ldz = ldz_for(V);
   const size_t es = elem_size(dtype);
   int64_t chunk = static_cast<int64_t>((ws_bytes - kWsHeader) / (static_cast<size_t>(ldz) * es)) / 128 * 128;
-  if (chunk >= N) chunk = N;
   if (chunk < 1) return PS_ERR_WORKSPACE;
+  // As few chunks as the workspace allows, of equal size (a multiple of 128 rows): a short last
+  // chunk would cost a whole pass over dW for little work.
+  const int64_t nchunks = (N + chunk - 1) / chunk;
+  chunk = ((N + nchunks - 1) / nchunks + 127) / 128 * 128;
+  if (chunk >= N) chunk = N;
   void* dz = static_cast<uint8_t*>(ws) + kWsHeader;
   for (int64_t r0 = 0; r0 < N; r0 += chunk) {
     const int64_t rcn = (N - r0) < chunk ? (N - r0) : chunk;
