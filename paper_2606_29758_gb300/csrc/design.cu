@@ -207,41 +207,70 @@ __global__ void group_offsets_kernel(int B, const int32_t* __restrict__ L, int64
 }
 
 // ================================================================== design
+// Lanes of the warp that tries saturated prefixes side by side in the capped design.
+constexpr int kCapLanes = 32;
+
 struct DesignWs {
   double* w;       // [P][T_max] weights
   double* xi;      // [P][T_max]
-  double* bW;      // [P][T_max] PAV block weights
-  int32_t* bn;     // [P][T_max] PAV block lengths
+  double* bW;      // [P][T_max][kCapLanes] PAV block weights, one stack per lane (interleaved)
+  double* bs;      // [P][T_max][kCapLanes] PAV block scores sqrt(W / n)
+  int32_t* bn;     // [P][T_max][kCapLanes] PAV block lengths
   int64_t* off;    // [P][K] row offsets of the group's completions
 };
 
-// Monotone design of w[0..T) with budget B into xi (Appendix F): pool adjacent violators while
-// sqrt(W_prev / n_prev) < sqrt(W_last / n_last), then xi_m = B s_m / sum_j n_j s_j.
-__device__ void monotone_design_dev(const double* w, int T, double B, double* xi, double* bW, int32_t* bn) {
+// True when the block (Wc, nc) violates the order against the block (Wp, np) below it, i.e. when
+// sqrt(Wp / np) < sqrt(Wc / nc) with both quotients and roots rounded to double, exactly as the
+// sequential definition decides it. The cross products Wp nc and Wc np settle every case whose
+// quotients differ by more than 2^-40 relative (then the rounded roots are ordered the same way);
+// only near-ties pay for the two divisions and square roots, which are slow in double precision.
+__device__ __forceinline__ bool pav_violates(double Wp, int np, double Wc, int nc) {
+  const double a = __dmul_rn(Wp, static_cast<double>(nc));
+  const double b = __dmul_rn(Wc, static_cast<double>(np));
+  if (a > 0x1p-900 && b > 0x1p-900 && a < 0x1p900 && b < 0x1p900) {
+    if (b > __dmul_rn(a, 1.0 + 0x1p-40)) return true;
+    if (b < __dmul_rn(a, 1.0 - 0x1p-40)) return false;
+  }
+  return __dsqrt_rn(__ddiv_rn(Wp, static_cast<double>(np))) < __dsqrt_rn(__ddiv_rn(Wc, static_cast<double>(nc)));
+}
+
+// Pool adjacent violators over w[0..T) (Appendix F) into one lane's stack (element m of the stack
+// at index m * kCapLanes): a new block is merged with the one below it while the block below has
+// the smaller score sqrt(W / n); merged weights add as W_prev + W_last, in the order of the
+// sequential definition, so every block sum is the same double. Returns the number of blocks.
+__device__ int pav_stack_dev(const double* w, int T, double* bW, int32_t* bn) {
+  // The top block stays in registers (Wt, nt); the blocks below it are in memory at [0, nb - 1).
+  // Memory is read only when a merge uncovers the block below.
   int nb = 0;
+  double Wt = 0.0;
+  int nt = 0;
+  double wnext = T > 0 ? w[0] : 0.0;
   for (int t = 0; t < T; ++t) {
-    bW[nb] = w[t];
-    bn[nb] = 1;
-    ++nb;
-    while (nb > 1 && __dsqrt_rn(__ddiv_rn(bW[nb - 2], static_cast<double>(bn[nb - 2]))) <
-                         __dsqrt_rn(__ddiv_rn(bW[nb - 1], static_cast<double>(bn[nb - 1])))) {
-      bn[nb - 2] += bn[nb - 1];
-      bW[nb - 2] = __dadd_rn(bW[nb - 2], bW[nb - 1]);
+    double Wc = wnext;
+    if (t + 1 < T) wnext = w[t + 1];
+    int nc = 1;
+    while (nb > 0 && pav_violates(Wt, nt, Wc, nc)) {
+      Wc = __dadd_rn(Wt, Wc);
+      nc += nt;
       --nb;
+      if (nb > 0) {
+        Wt = bW[(nb - 1) * kCapLanes];
+        nt = bn[(nb - 1) * kCapLanes];
+      }
     }
+    if (nb > 0) {
+      bW[(nb - 1) * kCapLanes] = Wt;
+      bn[(nb - 1) * kCapLanes] = nt;
+    }
+    Wt = Wc;
+    nt = nc;
+    ++nb;
   }
-  double den = 0.0;
-  for (int m = 0; m < nb; ++m) {
-    const double sm = __dsqrt_rn(__ddiv_rn(bW[m], static_cast<double>(bn[m])));
-    den = __dadd_rn(den, __dmul_rn(static_cast<double>(bn[m]), sm));
+  if (nb > 0) {
+    bW[(nb - 1) * kCapLanes] = Wt;
+    bn[(nb - 1) * kCapLanes] = nt;
   }
-  int t0 = 0;
-  for (int m = 0; m < nb; ++m) {
-    const double sm = __dsqrt_rn(__ddiv_rn(bW[m], static_cast<double>(bn[m])));
-    const double v = __ddiv_rn(__dmul_rn(B, sm), den);
-    for (int j = 0; j < bn[m]; ++j) xi[t0 + j] = v;
-    t0 += bn[m];
-  }
+  return nb;
 }
 
 constexpr int kDesignThreads = 256;
@@ -259,6 +288,9 @@ __global__ void __launch_bounds__(kDesignThreads)
   __shared__ long long red_l[kDesignThreads / 32];
   __shared__ int red_i[kDesignThreads / 32];
   __shared__ double lam_s;
+  __shared__ int found_s;
+  __shared__ int nb_s[kCapLanes];
+  __shared__ double den_s[kCapLanes];
   const int lane = tid & 31, wid = tid >> 5;
   double* w = ws.w + static_cast<int64_t>(p) * T_max;
   double* xi = ws.xi + static_cast<int64_t>(p) * T_max;
@@ -308,24 +340,88 @@ __global__ void __launch_bounds__(kDesignThreads)
     const double fl = __dmul_rn(1e-12, wm);
     for (int t = tid; t < Tp; t += kDesignThreads) w[t] = wm > 0.0 ? (w[t] > fl ? w[t] : fl) : 1.0;
     __syncthreads();
-    if (tid == 0) {
-      double* bW = ws.bW + static_cast<int64_t>(p) * T_max;
-      int32_t* bn = ws.bn + static_cast<int64_t>(p) * T_max;
-      if (strategy == PS_DESIGN_OPTIMIZED) {
-        // the smallest saturated prefix s whose suffix design starts at or below 1
-        int s = 0;
-        for (; s < Tp; ++s) {
-          monotone_design_dev(w + s, Tp - s, __dsub_rn(Bp, static_cast<double>(s)), xi + s, bW, bn);
-          if (xi[s] <= 1.0) break;
+    if (strategy == PS_DESIGN_OPTIMIZED) {
+      // The smallest saturated prefix s whose suffix design (budget B - s) starts at or below 1.
+      // The first round tries s = 0 alone; later rounds try 32 consecutive prefixes, one per lane
+      // of warp 0, each with its own stack. All threads then take the blocks' scores
+      // s_m = sqrt(W_m / n_m); each lane sums den = sum_m n_m s_m in block order, and the first
+      // lane (smallest s) whose design starts at or below 1 settles the search.
+      const int64_t sbase = static_cast<int64_t>(p) * T_max * kCapLanes;
+      double* bW = ws.bW + sbase;
+      double* bs = ws.bs + sbase;
+      int32_t* bn = ws.bn + sbase;
+      if (tid == 0) found_s = -1;
+      int base = 0;
+      for (int width = 1; base < Tp; base += width, width = kCapLanes) {
+        if (wid == 0) {
+          const int st = base + lane;
+          nb_s[lane] = (lane < width && st < Tp) ? pav_stack_dev(w + st, Tp - st, bW + lane, bn + lane) : 0;
         }
-        for (int t = 0; t < s && t < Tp; ++t) xi[t] = 1.0;
-      } else {
-        double tot = 0.0;
-        for (int t = 0; t < Tp; ++t) tot = __dadd_rn(tot, __dsqrt_rn(w[t]));
-        for (int t = 0; t < Tp; ++t) xi[t] = __ddiv_rn(__dmul_rn(Bp, __dsqrt_rn(w[t])), tot);
-        for (int t = 1; t < Tp; ++t) xi[t] = fmin(xi[t - 1], xi[t]);
-        for (int t = 0; t < Tp; ++t) xi[t] = fmin(xi[t], 1.0);
+        __syncthreads();
+        for (int l = 0; l < width; ++l)
+          for (int m = tid; m < nb_s[l]; m += kDesignThreads)
+            bs[m * kCapLanes + l] =
+                __dsqrt_rn(__ddiv_rn(bW[m * kCapLanes + l], static_cast<double>(bn[m * kCapLanes + l])));
+        __syncthreads();
+        if (wid == 0) {
+          const int st = base + lane;
+          bool ok = false;
+          if (lane < width && st < Tp) {
+            double den = 0.0;
+            for (int m = 0; m < nb_s[lane]; ++m)
+              den = __dadd_rn(den, __dmul_rn(static_cast<double>(bn[m * kCapLanes + lane]), bs[m * kCapLanes + lane]));
+            den_s[lane] = den;
+            ok = __ddiv_rn(__dmul_rn(__dsub_rn(Bp, static_cast<double>(st)), bs[lane]), den) <= 1.0;
+          }
+          const unsigned m = __ballot_sync(0xffffffffu, ok);
+          if (lane == 0 && m != 0u) found_s = base + __ffs(m) - 1;
+        }
+        __syncthreads();
+        if (found_s >= 0) break;
       }
+      const int found = found_s;
+      if (found < 0) {
+        for (int t = tid; t < Tp; t += kDesignThreads) xi[t] = 1.0;
+      } else {
+        // the design of lane l = found - base: block starts by a scan, then every block in parallel
+        const int l = found - base;
+        const int nb = nb_s[l];
+        const double Bs = __dsub_rn(Bp, static_cast<double>(found));
+        const double den = den_s[l];
+        for (int t = tid; t < found; t += kDesignThreads) xi[t] = 1.0;
+        if (tid == 0) {
+          int t0 = found;
+          for (int m = 0; m < nb; ++m) {
+            const int n = bn[m * kCapLanes + l];
+            bn[m * kCapLanes + l] = t0;          // the block's first step replaces its length
+            t0 += n;
+          }
+        }
+        __syncthreads();
+        for (int m = tid; m < nb; m += kDesignThreads) {
+          const double v = __ddiv_rn(__dmul_rn(Bs, bs[m * kCapLanes + l]), den);
+          const int t_end = m + 1 < nb ? bn[(m + 1) * kCapLanes + l] : Tp;
+          for (int t = bn[m * kCapLanes + l]; t < t_end; ++t) xi[t] = v;
+        }
+      }
+    } else {
+      // Heuristic: closed form B sqrt(w_t) / sum_j sqrt(w_j) (the sum in step order), a running
+      // minimum, then the cap at 1. The roots and quotients are taken in parallel.
+      for (int t = tid; t < Tp; t += kDesignThreads) xi[t] = __dsqrt_rn(w[t]);
+      __syncthreads();
+      if (tid == 0) {
+        double tot = 0.0;
+        for (int t = 0; t < Tp; ++t) tot = __dadd_rn(tot, xi[t]);
+        den_s[0] = tot;
+      }
+      __syncthreads();
+      const double tot = den_s[0];
+      for (int t = tid; t < Tp; t += kDesignThreads) xi[t] = __ddiv_rn(__dmul_rn(Bp, xi[t]), tot);
+      __syncthreads();
+      if (tid == 0)
+        for (int t = 1; t < Tp; ++t) xi[t] = fmin(xi[t - 1], xi[t]);
+      __syncthreads();
+      for (int t = tid; t < Tp; t += kDesignThreads) xi[t] = fmin(xi[t], 1.0);
     }
   } else if (strategy == PS_DESIGN_UNIFORM) {
     for (int t = tid; t < Tp; t += kDesignThreads)
@@ -352,6 +448,7 @@ __global__ void __launch_bounds__(kDesignThreads)
       for (int it = 0; it < 64 && budget_at(hi) > Bp; ++it) hi *= 2.0;
       for (int it = 0; it < 200; ++it) {
         const double mid = 0.5 * (lo + hi);
+        if (mid <= lo || mid >= hi) break;   // lo and hi are adjacent doubles: nothing changes any more
         if (budget_at(mid) > Bp) lo = mid;
         else hi = mid;
       }
@@ -512,9 +609,11 @@ static DesignWs design_ws(void* ws, int P, int K, int T_max) {
   d.xi = reinterpret_cast<double*>(b);
   b += al256(sizeof(double) * pt);
   d.bW = reinterpret_cast<double*>(b);
-  b += al256(sizeof(double) * pt);
+  b += al256(sizeof(double) * pt * kCapLanes);
+  d.bs = reinterpret_cast<double*>(b);
+  b += al256(sizeof(double) * pt * kCapLanes);
   d.bn = reinterpret_cast<int32_t*>(b);
-  b += al256(sizeof(int32_t) * pt);
+  b += al256(sizeof(int32_t) * pt * kCapLanes);
   d.off = reinterpret_cast<int64_t*>(b);
   return d;
 }
@@ -522,8 +621,8 @@ static DesignWs design_ws(void* ws, int P, int K, int T_max) {
 size_t ps_design_cutoffs_workspace_size(int P, int K, int T_max) {
   if (P < 1 || K < 1 || T_max < 1) return 0;
   const size_t pt = static_cast<size_t>(P) * T_max;
-  return kWsHeader + al256(sizeof(double) * pt) * 3 + al256(sizeof(int32_t) * pt) +
-         al256(sizeof(int64_t) * static_cast<size_t>(P) * K);
+  return kWsHeader + al256(sizeof(double) * pt) * 2 + al256(sizeof(double) * pt * kCapLanes) * 2 +
+         al256(sizeof(int32_t) * pt * kCapLanes) + al256(sizeof(int64_t) * static_cast<size_t>(P) * K);
 }
 
 int ps_design_cutoffs(int P, int K, int T_max, const int32_t* L, const float* gamma_full, const float* u,
