@@ -171,8 +171,10 @@ def run_ours(args):
     t1 = torch.cuda.Event(enable_timing=True)
     t0.record(stream)
     rows = 0
+    step_rows = []
     for i in range(args.steps):
-        rows += step(i, evs[i])
+        step_rows.append(step(i, evs[i]))
+        rows += step_rows[-1]
     t1.record(stream)
     barrier()
     clk = clocks.stop()
@@ -270,8 +272,9 @@ def run_ours(args):
     achieved_tf = fwd_flops / t_fwd / 1e12
     step_s = ms / args.steps * 1e-3
     credited_tf = 6.0 * mean_rows * d * V / step_s / 1e12
-    chunks = -(-int(round(mean_rows)) // args.chunk_rows)
-    launches_per_step = 1 + 2 + 3 + 3 * chunks
+    # per step: sampler 1, packing 2, forward 3 (GEMM, finalize, loss reduction), backward 3 per
+    # chunk (recompute, dH, dW); the backward splits a step's rows into ceil(N / chunk) chunks
+    launches = sum(6 + 3 * (-(-n // args.chunk_rows)) for n in step_rows)
     out = {
         "metric": "prefix tokens/s (fused LM-head PS-PPO fwd+bwd, 1xGB300)",
         "value": rows_all / (ms_max * 1e-3),
@@ -305,7 +308,7 @@ def run_ours(args):
                 "h2d_alone_ms": h2d_ms, "h2d_alone_gbs": h2d / (h2d_ms * 1e-3) / 1e9,
                 "overlap": "next batch copied on a second stream during the current pass (InputStager)"},
         "full_control": full_control,
-        "gpu_launches": launches_per_step * args.steps,
+        "gpu_launches": launches,
         "clocks": clk,
     }
     if design is not None:
