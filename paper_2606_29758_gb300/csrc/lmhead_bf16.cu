@@ -464,8 +464,9 @@ constexpr int kRecHalves = 1;
 
 // The forward keeps one band of row blocks in flight; every CTA re-reads its row block for
 // every vocabulary tile, so the band's hidden rows must stay in L2 (129 MB) next to the W
-// tiles being streamed: they get a third of it.
-constexpr double kFwdBandL2Bytes = 43e6;
+// tiles being streamed: they get about a quarter of it (30 MB measured 2% faster on the 7B-shaped
+// forward than 20 MB or 43 MB, and 64-86 MB were slower still).
+constexpr double kFwdBandL2Bytes = 30e6;
 
 static int fwd_band_max(int d) {
   const double block_bytes = static_cast<double>(kBM * kFwdHalves) * d * 2.0;
