@@ -194,9 +194,11 @@ int ps_lmhead_ppo_bwd(int64_t N, int d, int V, int dtype, const void* Hpk, const
  *
  * Appendix D: for a softmax head the squared norm of the head score is
  *   gamma_i = ||h_i||^2 (1 - 2 p_i(o_i) + ||p_i||^2),  p_i = softmax(W h_i),
- * with ||p||^2 = exp(LSE(2z) - 2 LSE(z)) (two logsumexp reductions). One pass of the head
- * GEMM over the rows (e.g. every token of the rollouts, with the old-policy head) gives
- * gamma [N] f32 and, if logp is not NULL, log p_i(o_i) [N] f32.
+ * i.e. ||h_i||^2 ||e_o - p_i||^2. The epilogue keeps two running sums over the row's
+ * logits other than the chosen one, r1 = sum_v e^(z_v - m) and r2 = sum_v e^(2 (z_v - m)),
+ * and evaluates ||e_o - p||^2 = (r1^2 + r2) / (e^(z_o - m) + r1)^2, which does not cancel as
+ * p(o) -> 1. One pass of the head GEMM over the rows (e.g. every token of the rollouts,
+ * with the old-policy head) gives gamma [N] f32 and, if logp is not NULL, log p_i(o_i) [N] f32.
  * Hrows [N][d] bf16, W [V][d] bf16 (bf16 only: other dtypes return PS_ERR_UNSUPPORTED),
  * tok [N] int32 (PS_DEV_BAD_TOKEN and NaN outputs for ids outside [0, V)).
  * topk (0..16): if > 0, the same pass also returns each row's topk most likely next tokens,
@@ -250,7 +252,8 @@ int ps_reward_uncertainty(int P, int K, int T_max, const int32_t* L, const float
  * deficit 2^62 - sum_h q[p][h-1] is Pr(H = 0): sample with PS_MODE_TRUNC_ZERO. xi [P][T_max]
  * f64 (may be NULL). Inputs: L [B] int32, gamma_full [sum L] f32 in completion order (needed
  * by OPTIMIZED and HEURISTIC, may be NULL otherwise), u [P][T_max] f32 or NULL.
- * All arithmetic is sequential f64, so the masses are reproducible bit for bit.
+ * The arithmetic is f64 in the order of the sequential definition (the parallel parts change
+ * no rounding), so the masses are reproducible bit for bit.
  * ------------------------------------------------------------------------- */
 enum {
   PS_DESIGN_OPTIMIZED = 0, PS_DESIGN_HEURISTIC = 1, PS_DESIGN_UNIFORM = 2,
