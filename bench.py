@@ -330,7 +330,11 @@ def run_ours(args):
     if design is not None:
         out["design_stage"] = design
     if rank == 0 and not args.no_cpu_baseline:
-        out["cpu_baseline"] = cpu_baseline(cfg, b, args.cpu_rows)
+        cb = cpu_baseline(cfg, b, args.cpu_rows)
+        # linear extrapolation from the sample to a whole step of mean_rows packed rows
+        cb["extrapolated_step_s"] = mean_rows / cb["value"]
+        cb["extrapolated_note"] = "extrapolated linearly from the sample to one step's packed rows"
+        out["cpu_baseline"] = cb
     if world > 1:
         dist.destroy_process_group()
     if rank == 0:
