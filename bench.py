@@ -350,39 +350,24 @@ def time_design_stage(cfg, b, dev, stream, reps=3):
     tokens, the reward-uncertainty proxy u_t per prompt and step, and the optimized design
     (closed form + PAV + cap, budget 128) into sampler masses."""
     import torch
-    from paper_2606_29758_gb300 import _binding as B
+    from paper_2606_29758_gb300 import CutoffDesign, DesignShape
     D = b.dev
     N = b.total_len
-    T = b.T_max
-    k = 16
-    gamma = torch.empty(N, device=dev)
-    logp = torch.empty(N, device=dev)
-    tidx = torch.empty(N, k, dtype=torch.int32, device=dev)
-    tprob = torch.empty(N, k, device=dev)
-    ws_p = torch.empty(B.ps_lmhead_score_proxy_workspace_size(N, cfg.d, cfg.V, B.PS_DTYPE_BF16, k), dtype=torch.uint8,
-                       device=dev)
-    u = torch.empty(cfg.P, T, device=dev)
-    ws_u = torch.empty(B.ps_reward_uncertainty_workspace_size(cfg.P, cfg.K), dtype=torch.uint8, device=dev)
-    q = torch.empty(cfg.P, T, dtype=torch.int64, device=dev)
-    ws_d = torch.empty(B.ps_design_cutoffs_workspace_size(cfg.P, cfg.K, T), dtype=torch.uint8, device=dev)
+    cd = CutoffDesign(DesignShape(cfg.P, cfg.K, b.T_max, cfg.d, cfg.V, N, 16), device=dev)
     ev = [torch.cuda.Event(enable_timing=True) for _ in range(4)]
     t = []
     for r in range(reps + 1):
         ev[0].record(stream)
-        B.ps_lmhead_score_proxy(N, cfg.d, cfg.V, B.PS_DTYPE_BF16, D["hid_full"], D["W"], D["tok_full"], gamma, logp,
-                                ws_p, k, tidx, tprob)
+        cd.score(D["hid_full"], D["W"], D["tok_full"])
         ev[1].record(stream)
-        B.ps_reward_uncertainty(cfg.P, cfg.K, T, D["L"], D["R"], k, tidx, tprob, u, ws_u)
+        cd.uncertainty(D["L"], D["R"])
         ev[2].record(stream)
-        B.ps_design_cutoffs(cfg.P, cfg.K, T, D["L"], gamma, u, 128.0, B.PS_DESIGN_OPTIMIZED, 0.0, q, None, ws_d)
+        cd.design(D["L"], 128.0)
         ev[3].record(stream)
         torch.cuda.synchronize()
         if r > 0:
             t.append([ev[i].elapsed_time(ev[i + 1]) for i in range(3)])
-    for ws in (ws_p, ws_u, ws_d):
-        rc, bits = B.ps_workspace_status(ws)
-        if rc != B.PS_OK:
-            raise B.PsppoError(rc, f"design stage (device bits {bits:#x})")
+    cd.check_status()
     pm, um, dm = (float(x) for x in np.mean(np.array(t), axis=0))
     return {"rows": N, "proxy_topk_ms": pm, "uncertainty_ms": um, "design_ms": dm,
             "proxy_tflops": 2.0 * N * cfg.d * cfg.V / (pm * 1e-3) / 1e12,

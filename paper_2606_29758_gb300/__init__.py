@@ -2,15 +2,16 @@
 
 The computation lives in libpsppo.so (hand-written CUDA, tcgen05 tensor cores, TMA)
 behind the C ABI of include/psppo.h; this package is its ctypes binding (same names)
-plus UpdatePass, which holds the device buffers of one batch shape in torch, and InputStager, which
-copies the next batch from host memory while the current one runs.
+plus UpdatePass, which holds the device buffers of one batch shape in torch, CutoffDesign, which
+does the same for the cutoff design upstream of it, and InputStager, which copies the next batch
+from host memory while the current one runs.
 """
 from ._binding import *  # noqa: F401,F403
 from ._binding import PsppoError, lib, status_string  # noqa: F401
 
 
 def __getattr__(name):
-    if name in ("UpdatePass", "PassShape", "InputStager"):
+    if name in ("UpdatePass", "PassShape", "InputStager", "CutoffDesign", "DesignShape"):
         from . import pipeline
         return getattr(pipeline, name)
     raise AttributeError(name)

@@ -146,3 +146,81 @@ class InputStager:
 
     def release(self, j: int, stream=None):
         self.free[j].record(stream or torch.cuda.current_stream())
+
+
+@dataclass
+class DesignShape:
+    P: int
+    K: int
+    T_max: int
+    d: int
+    V: int
+    rows: int                     # rollout tokens (sum of the completions' lengths)
+    topk: int = 16                # next tokens kept per rollout token for u_t (0: no u_t)
+
+
+class CutoffDesign:
+    """The cutoff design upstream of the update (Algorithm 1, steps 7-9), with buffers held in torch.
+
+    CutoffDesign owns the device buffers of one batch shape and runs, on the current stream:
+    the score proxy (and, with topk > 0, the top-k next tokens) of every rollout token under the
+    old-policy head; the reward-uncertainty proxy u_t per prompt and step; and the design of each
+    prompt's cutoff distribution into sampler masses `q` [P][T_max] (sample them with
+    PS_MODE_TRUNC_ZERO: a design may leave Pr(H = 0) > 0).
+    """
+
+    def __init__(self, shape: DesignShape, device: str = "cuda"):
+        s = shape
+        self.s, self.device = s, device
+        f32 = dict(dtype=torch.float32, device=device)
+        u8 = dict(dtype=torch.uint8, device=device)
+        self.gamma = torch.empty(s.rows, **f32)
+        self.logp = torch.empty(s.rows, **f32)
+        k = max(s.topk, 0)
+        self.top_idx = torch.empty(s.rows, max(k, 1), dtype=torch.int32, device=device)
+        self.top_prob = torch.empty(s.rows, max(k, 1), **f32)
+        self.u = torch.empty(s.P, s.T_max, **f32)
+        self.q = torch.zeros(s.P, s.T_max, dtype=torch.int64, device=device)
+        self.xi = torch.zeros(s.P, s.T_max, dtype=torch.float64, device=device)
+        self.ws_proxy = torch.zeros(B.ps_lmhead_score_proxy_workspace_size(s.rows, s.d, s.V, B.PS_DTYPE_BF16, k),
+                                    **u8)
+        self.ws_u = torch.zeros(B.ps_reward_uncertainty_workspace_size(s.P, s.K), **u8) if k > 0 else None
+        self.ws_design = torch.zeros(B.ps_design_cutoffs_workspace_size(s.P, s.K, s.T_max), **u8)
+
+    def score(self, hid_full, W_old, tok_full):
+        """gamma (and log p(o), and the top-k next tokens) of every rollout token."""
+        s = self.s
+        k = max(s.topk, 0)
+        B.ps_lmhead_score_proxy(s.rows, s.d, s.V, B.PS_DTYPE_BF16, hid_full, W_old, tok_full, self.gamma, self.logp,
+                                self.ws_proxy, k, self.top_idx if k else None, self.top_prob if k else None)
+
+    def uncertainty(self, L, R):
+        s = self.s
+        if s.topk <= 0:
+            raise ValueError("u_t needs the top-k next tokens (topk > 0)")
+        B.ps_reward_uncertainty(s.P, s.K, s.T_max, L, R, s.topk, self.top_idx, self.top_prob, self.u, self.ws_u)
+
+    def design(self, L, budget: float, strategy: int = B.PS_DESIGN_OPTIMIZED, param: float = 0.0,
+               use_u: bool = True):
+        s = self.s
+        B.ps_design_cutoffs(s.P, s.K, s.T_max, L, self.gamma, self.u if (use_u and s.topk > 0) else None, budget,
+                            strategy, param, self.q, self.xi, self.ws_design)
+
+    def run(self, hid_full, W_old, tok_full, L, R, budget: float, strategy: int = B.PS_DESIGN_OPTIMIZED,
+            param: float = 0.0):
+        """Proxy -> u_t -> design; returns the masses q."""
+        if strategy in (B.PS_DESIGN_OPTIMIZED, B.PS_DESIGN_HEURISTIC):
+            self.score(hid_full, W_old, tok_full)
+            if self.s.topk > 0:
+                self.uncertainty(L, R)
+        self.design(L, budget, strategy, param)
+        return self.q
+
+    def check_status(self):
+        """Raise PsppoError if any workspace reports a device-side error."""
+        for name, ws in (("proxy", self.ws_proxy), ("uncertainty", self.ws_u), ("design", self.ws_design)):
+            if ws is None:
+                continue
+            rc, bits = B.ps_workspace_status(ws)
+            if rc != B.PS_OK:
+                raise B.PsppoError(rc, f"{name} (device bits {bits:#x})")

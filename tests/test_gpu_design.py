@@ -235,3 +235,36 @@ def test_design_then_update_end_to_end():
     assert torch.isfinite(up.loss).all() and torch.isfinite(up.dH[:Nr]).all() and torch.isfinite(up.dW).all()
     # weights are 1/xi of the realised distribution
     assert float(up.w[:Nr].min()) >= 1.0
+
+
+def test_cutoff_design_holder_matches_the_abi_calls():
+    # CutoffDesign runs the same three calls; its masses equal those of the calls made one by one
+    from paper_2606_29758_gb300 import _binding as B
+    from paper_2606_29758_gb300 import CutoffDesign, DesignShape
+    cfg = get_config("mid")
+    b = make_batch(cfg, device="cuda")
+    D = b.dev
+    N, T, k = b.total_len, b.T_max, 16
+    cd = CutoffDesign(DesignShape(cfg.P, cfg.K, T, cfg.d, cfg.V, N, k))
+    q = cd.run(D["hid_full"], D["W"], D["tok_full"], D["L"], D["R"], 40.0).clone()
+    gamma = torch.empty(N, device="cuda")
+    tidx = torch.empty(N, k, dtype=torch.int32, device="cuda")
+    tprob = torch.empty(N, k, device="cuda")
+    ws_p = torch.zeros(B.ps_lmhead_score_proxy_workspace_size(N, cfg.d, cfg.V, B.PS_DTYPE_BF16, k),
+                       dtype=torch.uint8, device="cuda")
+    B.ps_lmhead_score_proxy(N, cfg.d, cfg.V, B.PS_DTYPE_BF16, D["hid_full"], D["W"], D["tok_full"], gamma, None,
+                            ws_p, k, tidx, tprob)
+    u = torch.empty(cfg.P, T, device="cuda")
+    ws_u = torch.zeros(B.ps_reward_uncertainty_workspace_size(cfg.P, cfg.K), dtype=torch.uint8, device="cuda")
+    B.ps_reward_uncertainty(cfg.P, cfg.K, T, D["L"], D["R"], k, tidx, tprob, u, ws_u)
+    q2 = torch.zeros(cfg.P, T, dtype=torch.int64, device="cuda")
+    ws_d = torch.zeros(B.ps_design_cutoffs_workspace_size(cfg.P, cfg.K, T), dtype=torch.uint8, device="cuda")
+    B.ps_design_cutoffs(cfg.P, cfg.K, T, D["L"], gamma, u, 40.0, B.PS_DESIGN_OPTIMIZED, 0.0, q2, None, ws_d)
+    torch.cuda.synchronize()
+    cd.check_status()
+    assert torch.equal(q, q2) and torch.equal(cd.gamma, gamma) and torch.equal(cd.u, u)
+    # the other strategies through the holder, checked against the oracle's masses
+    for strategy, name, param in ((B.PS_DESIGN_UNIFORM, "uniform", 0.0), (B.PS_DESIGN_FIXED, "fixed", 12.0)):
+        qs = cd.run(D["hid_full"], D["W"], D["tok_full"], D["L"], D["R"], 40.0, strategy, param).cpu().numpy()
+        q_ref, _ = design.design_cutoff_masses(b.L, cfg.K, np.zeros(N, np.float32), None, 40.0, name, param=param)
+        assert np.array_equal(qs.view(np.uint64), q_ref), name
