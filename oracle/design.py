@@ -302,3 +302,47 @@ def reward_uncertainty(L, K, R, top_idx, top_prob):
             l1 = sum(abs(x) for x in mass.values()) + abs(other)
             u[p, t] = min(0.5, max(0.0, 0.5 - 0.5 * l1))
     return u
+
+
+# ---------------------------------------------------------------- continuous rewards (Appendix G)
+LN2 = 0.6931471805599453          # the double nearest ln 2
+SIGMOID_CLAMP = 40.0              # |r| beyond this decides no label differently (see below)
+
+
+def sigmoid_recipe(r: float) -> float:
+    """sigma(r) = 1 / (1 + e^(-r)) by one fixed sequence of IEEE double operations.
+
+    With z = -r clamped to [-40, 40]: k = floor(z / ln2 + 1/2), f = z - k ln2 (|f| <= ln2 / 2 plus
+    rounding), e^f by Horner's rule over its Taylor series to degree 16 (p <- 1 + f p / n for
+    n = 16, ..., 1; the truncation error is below 1e-22), e^z = e^f 2^k, and sigma = 1 / (1 + e^z).
+    Every step is a correctly rounded +, -, *, / or an exact power-of-two scaling, so the kernel
+    that repeats the sequence gets the same double. The clamp moves sigma by less than 4.3e-18,
+    below the 2^-53 resolution of the uniform it is compared with, so no label changes.
+    """
+    r = float(r)
+    if r != r:
+        return 0.0
+    z = -r
+    z = SIGMOID_CLAMP if z > SIGMOID_CLAMP else (-SIGMOID_CLAMP if z < -SIGMOID_CLAMP else z)
+    k = math.floor(z / LN2 + 0.5)
+    f = z - k * LN2
+    p = 1.0
+    for n in range(16, 0, -1):
+        p = 1.0 + (f * p) / n
+    e = math.ldexp(p, k)
+    return 1.0 / (1.0 + e)
+
+
+def binarize_rewards(R, seed: int, step: int, traj_base: int = 0) -> np.ndarray:
+    """Appendix G: labels y_k ~ Bernoulli(sigma(R_k)) for the u_t estimate only (the update keeps
+    the continuous R). Trajectory k draws u = m 2^-53 from the Philox stream keyed by
+    (seed, "PSPPRWD1") at counter (traj_base + k, step, 0, 0), and y_k = 1 when u < sigma(R_k),
+    i.e. when m < sigma 2^53 (a NaN reward gives 0). Returns float32 labels in {0, 1}.
+    """
+    from .philox import reward_uniform53
+    R = np.asarray(R, dtype=np.float32)
+    y = np.zeros(len(R), dtype=np.float32)
+    for k, r in enumerate(R):
+        m = reward_uniform53(seed, step, traj_base + k)
+        y[k] = 1.0 if float(m) < sigmoid_recipe(float(r)) * 9007199254740992.0 else 0.0
+    return y

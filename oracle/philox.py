@@ -46,3 +46,17 @@ def cutoff_uniform62(seed: int, step: int, traj: int) -> int:
     """
     out = philox4x64_10((traj, step, 0, 0), (seed, CUTOFF_KEY_TAG))
     return out[0] >> 2
+
+
+# Key word 1 of the reward-binarisation stream: the ASCII bytes "PSPPRWD1".
+REWARD_KEY_TAG = 0x5053505052574431
+
+
+def reward_uniform53(seed: int, step: int, traj: int) -> int:
+    """The 53-bit uniform integer that binarises trajectory `traj`'s reward for u_t.
+
+    key = (seed, "PSPPRWD1"), counter = (global trajectory index, step, 0, 0); the first output
+    word shifted right by 11 is uniform on [0, 2^53), i.e. u = k 2^-53 on [0, 1).
+    """
+    out = philox4x64_10((traj, step, 0, 0), (seed, REWARD_KEY_TAG))
+    return out[0] >> 11

@@ -212,3 +212,38 @@ def test_topk_policy_orders_and_ties():
     idx, p = design.topk_policy(np.array([[1.0]]), W, 3)
     assert list(idx[0]) == [1, 2, 0]
     assert p[0, 0] == pytest.approx(p[0, 1]) and p[0].sum() < 1.0
+
+
+def test_sigmoid_recipe_is_the_logistic_function():
+    # Appendix G's sigma(r) = 1 / (1 + e^-r): against the library exponential, its symmetry and
+    # its fixed points
+    r = np.linspace(-40.0, 40.0, 40001)
+    got = np.array([design.sigmoid_recipe(x) for x in r])
+    ref = 1.0 / (1.0 + np.exp(-r))
+    assert np.max(np.abs(got - ref) / ref) < 1e-14
+    assert np.max(np.abs(got + got[::-1] - 1.0)) < 4e-15          # sigma(-r) = 1 - sigma(r)
+    assert np.all(np.diff(got) >= 0.0)
+    assert design.sigmoid_recipe(0.0) == 0.5
+    assert design.sigmoid_recipe(float("inf")) == design.sigmoid_recipe(1e9) == design.sigmoid_recipe(40.0)
+    assert design.sigmoid_recipe(float("nan")) == 0.0
+
+
+@pytest.mark.parametrize("r", [-3.0, -0.5, 0.0, 0.8, 2.5])
+def test_binarized_labels_are_bernoulli_sigma(r):
+    # y ~ Bernoulli(sigma(r)): the label frequency over many trajectories is sigma(r)
+    M = 4000
+    y = design.binarize_rewards(np.full(M, r, dtype=np.float32), seed=11, step=2)
+    assert set(np.unique(y)) <= {0.0, 1.0}
+    p = 1.0 / (1.0 + math.exp(-r))
+    assert abs(y.mean() - p) < 4.5 * math.sqrt(p * (1 - p) / M)
+
+
+def test_binarized_labels_extremes_and_streams():
+    y = design.binarize_rewards(np.array([60.0, -60.0, np.inf, -np.inf, np.nan], dtype=np.float32), 1, 0)
+    assert list(y[:1]) == [1.0] and y[2] == 1.0 and y[4] == 0.0
+    assert y[1] == 0.0 and y[3] == 0.0        # a label 1 would need the uniform to be exactly 0
+    # a shard starting at trajectory 7 draws what the whole batch draws for its trajectories
+    R = np.random.default_rng(0).normal(0, 2, 20).astype(np.float32)
+    whole = design.binarize_rewards(R, 5, 3)
+    assert np.array_equal(design.binarize_rewards(R[7:], 5, 3, traj_base=7), whole[7:])
+    assert not np.array_equal(design.binarize_rewards(R, 5, 4), whole)    # the step changes the draw

@@ -34,3 +34,14 @@ def test_cutoff_stream_matches_numpy():
                 ref = _numpy_block((k, step, 0, 0), (seed, CUTOFF_KEY_TAG))[0] >> 2
                 assert cutoff_uniform62(seed, step, k) == ref
                 assert 0 <= ref < (1 << 62)
+
+
+def test_reward_stream_matches_numpy():
+    from oracle.philox import REWARD_KEY_TAG, reward_uniform53
+    assert REWARD_KEY_TAG != CUTOFF_KEY_TAG
+    for seed in (0, 3, 2**64 - 1):
+        for step in (0, 9):
+            for k in range(1, 30):
+                ref = _numpy_block((k, step, 0, 0), (seed, REWARD_KEY_TAG))[0] >> 11
+                assert reward_uniform53(seed, step, k) == ref
+                assert 0 <= ref < (1 << 53)
