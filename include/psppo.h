@@ -227,6 +227,23 @@ int ps_lmhead_score_proxy(int64_t N, int d, int V, int dtype, const void* Hrows,
  * f32 in completion order (as from ps_lmhead_score_proxy). Limits: K <= 64, 1 <= topk <= 16.
  * ------------------------------------------------------------------------- */
 size_t ps_reward_uncertainty_workspace_size(int P, int K);
+
+/* ---------------------------------------------------------------------------
+ * ps_binarize_rewards -- binary labels of continuous rewards, for u_t only.
+ *
+ * Appendix G: to use the u_t estimate with a continuous reward r, each completion's reward is
+ * turned into a label y ~ Bernoulli(sigma(r)), sigma(r) = 1 / (1 + e^-r); the labels feed
+ * ps_reward_uncertainty (as R), while the update keeps the continuous rewards. Completion k
+ * (global index traj_base + k) draws u = m 2^-53 from Philox4x64-10 with key (seed,
+ * 0x5053505052574431 "PSPPRWD1") and counter (traj_base + k, step, 0, 0), m = first output
+ * word >> 11, and y_k = 1 if u < sigma(R_k), else 0 (a NaN reward gives 0). sigma is taken by
+ * a fixed sequence of double operations (|r| clamped to 40, exp by range reduction and a
+ * degree-16 Taylor polynomial), so the labels are reproducible bit for bit. Binary rewards
+ * in {0, 1} need no binarisation: pass them to ps_reward_uncertainty directly.
+ * R [B] f32 in, y [B] f32 out (0 or 1). No workspace; asynchronous on `stream`.
+ * ------------------------------------------------------------------------- */
+int ps_binarize_rewards(int B, const float* R, uint64_t seed, uint64_t step, int64_t traj_base,
+                        float* y, ps_stream_t stream);
 int ps_reward_uncertainty(int P, int K, int T_max, const int32_t* L, const float* R, int topk,
                           const int32_t* top_idx, const float* top_prob, float* u,
                           void* ws, size_t ws_bytes, ps_stream_t stream);

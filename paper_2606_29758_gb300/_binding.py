@@ -31,7 +31,7 @@ EXPORTS = [
     "ps_diag_gemm_bf16", "ps_diag_wait_timeout", "ps_lmhead_ppo_fwd_noalloc",
     "ps_lmhead_score_proxy_workspace_size", "ps_lmhead_score_proxy",
     "ps_design_cutoffs_workspace_size", "ps_design_cutoffs",
-    "ps_reward_uncertainty_workspace_size", "ps_reward_uncertainty",
+    "ps_reward_uncertainty_workspace_size", "ps_reward_uncertainty", "ps_binarize_rewards",
 ]
 PS_DESIGN_OPTIMIZED, PS_DESIGN_HEURISTIC, PS_DESIGN_UNIFORM, PS_DESIGN_TIME_PRIOR, PS_DESIGN_FIXED = range(5)
 
@@ -81,6 +81,7 @@ _SIGS = {
                                      _vp]),
     "ps_reward_uncertainty_workspace_size": (_sz, [_i32, _i32]),
     "ps_reward_uncertainty": (_i32, [_i32, _i32, _i32, _vp, _vp, _i32, _vp, _vp, _vp, _vp, _sz, _vp]),
+    "ps_binarize_rewards": (_i32, [_i32, _vp, _u64, _u64, _i64, _vp, _vp]),
     "ps_design_cutoffs_workspace_size": (_sz, [_i32, _i32, _i32]),
     "ps_design_cutoffs": (_i32, [_i32, _i32, _i32, _vp, _vp, _vp, _f64, _i32, _f64, _vp, _vp, _vp, _sz, _vp]),
     "ps_lmhead_ppo_fwd_noalloc": (_i32, [_i64, _i32, _i32, _i32, _vp, _vp, _vp, _vp, _vp, _vp, _f64, _f64,
@@ -223,6 +224,11 @@ def ps_reward_uncertainty(P, K, T_max, L, R, topk, top_idx, top_prob, u, ws, str
     rc = lib().ps_reward_uncertainty(P, K, T_max, _ptr(L), _ptr(R), topk, _ptr(top_idx), _ptr(top_prob), _ptr(u),
                                      _ptr(ws), _nbytes(ws), _stream(stream))
     _check(rc, "ps_reward_uncertainty")
+
+
+def ps_binarize_rewards(B, R, seed, step, y, traj_base=0, stream=None):
+    rc = lib().ps_binarize_rewards(B, _ptr(R), seed, step, traj_base, _ptr(y), _stream(stream))
+    _check(rc, "ps_binarize_rewards")
 
 
 def ps_design_cutoffs_workspace_size(P: int, K: int, T_max: int) -> int:

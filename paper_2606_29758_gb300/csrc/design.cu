@@ -509,6 +509,40 @@ __global__ void __launch_bounds__(kDesignThreads)
   }
 }
 
+// ---------------------------------------------------------------- reward binarisation (Appendix G)
+constexpr uint64_t kRewardKeyTag = 0x5053505052574431ull;  // "PSPPRWD1"
+constexpr double kLn2d = 0.6931471805599453;              // the double nearest ln 2
+constexpr double kTwo53 = 9007199254740992.0;
+
+// sigma(r) = 1 / (1 + e^-r) by one fixed sequence of correctly rounded double operations:
+// z = -r clamped to [-40, 40], k = floor(z / ln2 + 1/2), f = z - k ln2, e^f by Horner's rule
+// over its Taylor series to degree 16, e^z = e^f 2^k (exact scaling), sigma = 1 / (1 + e^z).
+// No step is left to the compiler's choice (no contraction into FMAs), so the value is the
+// same double wherever the sequence is repeated. The clamp moves sigma by less than 4.3e-18.
+__device__ double sigmoid_fixed_dev(double r) {
+  if (r != r) return 0.0;
+  double z = -r;
+  z = z > 40.0 ? 40.0 : (z < -40.0 ? -40.0 : z);
+  const double k = floor(__dadd_rn(__ddiv_rn(z, kLn2d), 0.5));
+  const double f = __dsub_rn(z, __dmul_rn(k, kLn2d));
+  double p = 1.0;
+  for (int n = 16; n >= 1; --n) p = __dadd_rn(1.0, __ddiv_rn(__dmul_rn(f, p), static_cast<double>(n)));
+  const double two_k = __longlong_as_double(static_cast<long long>(static_cast<int>(k) + 1023) << 52);
+  return __ddiv_rn(1.0, __dadd_rn(1.0, __dmul_rn(p, two_k)));
+}
+
+// y_k = 1 when the trajectory's 53-bit Philox uniform lies below sigma(R_k), else 0.
+__global__ void binarize_rewards_kernel(int B, const float* __restrict__ R, uint64_t seed, uint64_t step,
+                                        int64_t traj_base, float* __restrict__ y) {
+  const int k = blockIdx.x * blockDim.x + threadIdx.x;
+  if (k >= B) return;
+  uint64_t c[4] = {static_cast<uint64_t>(traj_base + k), step, 0ull, 0ull};
+  philox4x64_10(c, seed, kRewardKeyTag);
+  const double m = static_cast<double>(c[0] >> 11);
+  const double s = sigmoid_fixed_dev(static_cast<double>(R[k]));
+  y[k] = m < __dmul_rn(s, kTwo53) ? 1.0f : 0.0f;
+}
+
 }  // namespace psk
 
 using namespace psk;
@@ -575,6 +609,14 @@ int ps_lmhead_score_proxy(int64_t N, int d, int V, int dtype, const void* Hrows,
 size_t ps_reward_uncertainty_workspace_size(int P, int K) {
   if (P < 1 || K < 1) return 0;
   return kWsHeader + al256(sizeof(int64_t) * static_cast<size_t>(P) * K);
+}
+
+int ps_binarize_rewards(int B, const float* R, uint64_t seed, uint64_t step, int64_t traj_base, float* y,
+                        ps_stream_t stream) {
+  if (B < 1 || traj_base < 0 || !R || !y) return PS_ERR_INVALID_ARG;
+  cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
+  binarize_rewards_kernel<<<(B + 255) / 256, 256, 0, s>>>(B, R, seed, step, traj_base, y);
+  return cudaGetLastError() == cudaSuccess ? PS_OK : PS_ERR_CUDA;
 }
 
 int ps_reward_uncertainty(int P, int K, int T_max, const int32_t* L, const float* R, int topk,

@@ -41,26 +41,6 @@ static int begin_call(void* ws, size_t ws_bytes, size_t need, cudaStream_t s) {
 
 static uint32_t* status_word(void* ws) { return static_cast<uint32_t*>(ws); }
 
-// ================================================================== philox4x64-10
-// Salmon et al., "Parallel Random Numbers: As Easy as 1, 2, 3" (SC'11).
-__device__ __forceinline__ void philox4x64_10(uint64_t (&c)[4], uint64_t k0, uint64_t k1) {
-  const uint64_t M0 = 0xD2E7470EE14C6C93ull, M1 = 0xCA5A826395121157ull;
-  const uint64_t W0 = 0x9E3779B97F4A7C15ull, W1 = 0xBB67AE8584CAA73Bull;
-#pragma unroll
-  for (int r = 0; r < 10; ++r) {
-    if (r > 0) {
-      k0 += W0;
-      k1 += W1;
-    }
-    const uint64_t lo0 = M0 * c[0], hi0 = __umul64hi(M0, c[0]);
-    const uint64_t lo1 = M1 * c[2], hi1 = __umul64hi(M1, c[2]);
-    const uint64_t n0 = hi1 ^ c[1] ^ k0, n2 = hi0 ^ c[3] ^ k1;
-    c[0] = n0;
-    c[1] = lo1;
-    c[2] = n2;
-    c[3] = lo0;
-  }
-}
 constexpr uint64_t kCutoffKeyTag = 0x5053505030303031ull;  // "PSPP0001"
 
 // ================================================================== K1: cutoff sampler

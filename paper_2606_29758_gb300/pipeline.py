@@ -180,6 +180,7 @@ class CutoffDesign:
         self.top_idx = torch.empty(s.rows, max(k, 1), dtype=torch.int32, device=device)
         self.top_prob = torch.empty(s.rows, max(k, 1), **f32)
         self.u = torch.empty(s.P, s.T_max, **f32)
+        self.y = torch.empty(s.P * s.K, **f32)          # reward labels for u_t (continuous rewards)
         self.q = torch.zeros(s.P, s.T_max, dtype=torch.int64, device=device)
         self.xi = torch.zeros(s.P, s.T_max, dtype=torch.float64, device=device)
         self.ws_proxy = torch.zeros(B.ps_lmhead_score_proxy_workspace_size(s.rows, s.d, s.V, B.PS_DTYPE_BF16, k),
@@ -194,11 +195,18 @@ class CutoffDesign:
         B.ps_lmhead_score_proxy(s.rows, s.d, s.V, B.PS_DTYPE_BF16, hid_full, W_old, tok_full, self.gamma, self.logp,
                                 self.ws_proxy, k, self.top_idx if k else None, self.top_prob if k else None)
 
-    def uncertainty(self, L, R):
+    def uncertainty(self, L, R, continuous: bool = False, seed: int = 0, step: int = 0, traj_base: int = 0):
+        """u_t per prompt and step. With continuous rewards, each is first turned into a label
+        y ~ Bernoulli(sigma(R)) (Appendix G; ps_binarize_rewards) used for u_t only."""
         s = self.s
         if s.topk <= 0:
             raise ValueError("u_t needs the top-k next tokens (topk > 0)")
-        B.ps_reward_uncertainty(s.P, s.K, s.T_max, L, R, s.topk, self.top_idx, self.top_prob, self.u, self.ws_u)
+        labels = R
+        if continuous:
+            B.ps_binarize_rewards(s.P * s.K, R, seed, step, self.y, traj_base)
+            labels = self.y
+        B.ps_reward_uncertainty(s.P, s.K, s.T_max, L, labels, s.topk, self.top_idx, self.top_prob, self.u,
+                                self.ws_u)
 
     def design(self, L, budget: float, strategy: int = B.PS_DESIGN_OPTIMIZED, param: float = 0.0,
                use_u: bool = True):
@@ -207,12 +215,12 @@ class CutoffDesign:
                             strategy, param, self.q, self.xi, self.ws_design)
 
     def run(self, hid_full, W_old, tok_full, L, R, budget: float, strategy: int = B.PS_DESIGN_OPTIMIZED,
-            param: float = 0.0):
+            param: float = 0.0, continuous: bool = False, seed: int = 0, step: int = 0):
         """Proxy -> u_t -> design; returns the masses q."""
         if strategy in (B.PS_DESIGN_OPTIMIZED, B.PS_DESIGN_HEURISTIC):
             self.score(hid_full, W_old, tok_full)
             if self.s.topk > 0:
-                self.uncertainty(L, R)
+                self.uncertainty(L, R, continuous, seed, step)
         self.design(L, budget, strategy, param)
         return self.q
 

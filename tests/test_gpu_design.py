@@ -268,3 +268,39 @@ def test_cutoff_design_holder_matches_the_abi_calls():
         qs = cd.run(D["hid_full"], D["W"], D["tok_full"], D["L"], D["R"], 40.0, strategy, param).cpu().numpy()
         q_ref, _ = design.design_cutoff_masses(b.L, cfg.K, np.zeros(N, np.float32), None, 40.0, name, param=param)
         assert np.array_equal(qs.view(np.uint64), q_ref), name
+
+
+def test_binarized_rewards_bit_exact_and_u_from_them():
+    # Appendix G: labels y ~ Bernoulli(sigma(R)) equal the oracle's bit for bit (same Philox
+    # stream, same fixed sigma sequence), and u_t from them matches the oracle's u_t
+    from paper_2606_29758_gb300 import _binding as B
+    from paper_2606_29758_gb300 import CutoffDesign, DesignShape
+    rng = np.random.default_rng(8)
+    R = np.concatenate([rng.normal(0.0, 2.0, 4000), [0.0, 40.0, -40.0, 60.0, -60.0, np.inf, -np.inf, np.nan],
+                        rng.uniform(-0.01, 0.01, 88)]).astype(np.float32)
+    Rd = torch.from_numpy(R).cuda()
+    y = torch.empty_like(Rd)
+    for seed, step, base in ((0, 0, 0), (7, 3, 0), (2**64 - 1, 2**40, 12345)):
+        B.ps_binarize_rewards(len(R), Rd, seed, step, y, base)
+        torch.cuda.synchronize()
+        ref = design.binarize_rewards(R, seed, step, traj_base=base)
+        assert np.array_equal(y.cpu().numpy(), ref), (seed, step)
+    # u_t through CutoffDesign with continuous rewards: seeded top-16 lists over a small shared
+    # vocabulary (as in the u_t test above) go into the holder's buffers, so both sides see the
+    # same inputs
+    cfg = get_config("mid")
+    L = draw_lengths(cfg)
+    N, k, T = int(L.sum()), 16, int(L.max())
+    idx = np.stack([rng.choice(64, size=k, replace=False) for _ in range(N)]).astype(np.int32)
+    prob = rng.dirichlet(np.ones(k + 1), size=N)[:, :k].astype(np.float32)
+    Rc = rng.normal(0.0, 1.5, cfg.B).astype(np.float32)       # continuous rewards
+    cd = CutoffDesign(DesignShape(cfg.P, cfg.K, T, cfg.d, cfg.V, N, k))
+    cd.top_idx.copy_(torch.from_numpy(idx))
+    cd.top_prob.copy_(torch.from_numpy(prob))
+    cd.uncertainty(torch.from_numpy(L).cuda(), torch.from_numpy(Rc).cuda(), continuous=True, seed=4, step=1)
+    torch.cuda.synchronize()
+    cd.check_status()
+    labels = design.binarize_rewards(Rc, 4, 1)
+    assert np.array_equal(cd.y.cpu().numpy(), labels)
+    u_ref = design.reward_uncertainty(L, cfg.K, labels, idx, prob)
+    np.testing.assert_allclose(cd.u.cpu().numpy(), u_ref, atol=2e-7)
