@@ -199,6 +199,17 @@ def run_ours(args):
         ms, step_rows, per, clk = timed_region(500)
         clk["remeasured_after"] = first.get("reasons", [])
     rows = sum(step_rows)
+    # the last timed step's rows: how many the clip switched off (coef = 0 with A != 0), and the
+    # packing rate (hidden rows read and written; the pack call includes its host sync)
+    n_last = step_rows[-1]
+    coef_last, adv_last = up.coef[:n_last], up.adv[:n_last]
+    clipped = int(((coef_last == 0) & (adv_last != 0)).sum().item())
+    pass_stats = {"rows_last_step": n_last, "clip_fraction": clipped / max(n_last, 1),
+                  "zero_advantage_fraction": float((adv_last == 0).float().mean().item()),
+                  "pack_gbs": 2.0 * float(np.mean(step_rows)) * cfg.d * (2 if cfg.dtype == "bf16" else 4)
+                  / (float(per[:, 1].mean()) * 1e-3) / 1e9,
+                  "sample_us": float(per[:, 0].mean()) * 1e3}
+
     ms_max = ms
     rows_all = rows
     if world > 1:
@@ -317,6 +328,7 @@ def run_ours(args):
         "per_call_ms": {"sample": float(per[:, 0].mean()), "pack": float(per[:, 1].mean()),
                         "fwd": float(per[:, 2].mean()), "bwd": float(per[:, 3].mean()),
                         "note": "pack includes its one host synchronisation (reading N)"},
+        "pass_stats": pass_stats,
         "roofline": {"kernel": "umma_gemm_kernel<K,K,FwdLseEpi> (fused forward; + O(N) finalize)",
                      "bound": "tensor", "achieved": achieved_tf, "peak": peak_tf, "unit": "TFLOP/s",
                      "frac": achieved_tf / peak_tf, "traffic": FWD_GEMM_TRAFFIC.get(cfg.name),

@@ -18,6 +18,7 @@
 #include <climits>
 #include <cstdint>
 
+#include "ps_nvtx.h"
 #include "internal.h"
 #include "ps_common.cuh"
 #include "psppo.h"
@@ -568,6 +569,7 @@ size_t ps_lmhead_score_proxy_workspace_size(int64_t N, int d, int V, int dtype, 
 int ps_lmhead_score_proxy(int64_t N, int d, int V, int dtype, const void* Hrows, const void* W, const int32_t* tok,
                           float* gamma, float* logp, int topk, int32_t* top_idx, float* top_prob, void* ws,
                           size_t ws_bytes, ps_stream_t stream) {
+  NvtxRange nvtx_range("ps_lmhead_score_proxy");
   if (N < 0 || N > INT32_MAX || V < 1 || d < 8 || d % 8 || topk < 0 || topk > 16) return PS_ERR_INVALID_ARG;
   if (dtype != PS_DTYPE_BF16) return PS_ERR_UNSUPPORTED;
   if (N > 0 && (!Hrows || !W || !tok || !gamma)) return PS_ERR_INVALID_ARG;
@@ -613,6 +615,7 @@ size_t ps_reward_uncertainty_workspace_size(int P, int K) {
 
 int ps_binarize_rewards(int B, const float* R, uint64_t seed, uint64_t step, int64_t traj_base, float* y,
                         ps_stream_t stream) {
+  NvtxRange nvtx_range("ps_binarize_rewards");
   if (B < 1 || traj_base < 0 || !R || !y) return PS_ERR_INVALID_ARG;
   cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
   binarize_rewards_kernel<<<(B + 255) / 256, 256, 0, s>>>(B, R, seed, step, traj_base, y);
@@ -622,6 +625,7 @@ int ps_binarize_rewards(int B, const float* R, uint64_t seed, uint64_t step, int
 int ps_reward_uncertainty(int P, int K, int T_max, const int32_t* L, const float* R, int topk,
                           const int32_t* top_idx, const float* top_prob, float* u, void* ws, size_t ws_bytes,
                           ps_stream_t stream) {
+  NvtxRange nvtx_range("ps_reward_uncertainty");
   if (P < 1 || K < 1 || K > 64 || T_max < 1 || topk < 1 || topk > 16) return PS_ERR_INVALID_ARG;
   if (!L || !R || !top_idx || !top_prob || !u) return PS_ERR_INVALID_ARG;
   if (ws == nullptr || (reinterpret_cast<uintptr_t>(ws) & 255) ||
@@ -670,6 +674,7 @@ size_t ps_design_cutoffs_workspace_size(int P, int K, int T_max) {
 int ps_design_cutoffs(int P, int K, int T_max, const int32_t* L, const float* gamma_full, const float* u,
                       double budget, int strategy, double param, uint64_t* q, double* xi, void* ws, size_t ws_bytes,
                       ps_stream_t stream) {
+  NvtxRange nvtx_range("ps_design_cutoffs");
   if (P < 1 || K < 1 || T_max < 1 || T_max > (1 << 24) || !L || !q) return PS_ERR_INVALID_ARG;
   if (static_cast<int64_t>(P) * K > INT32_MAX) return PS_ERR_INVALID_ARG;
   if (strategy < PS_DESIGN_OPTIMIZED || strategy > PS_DESIGN_FIXED) return PS_ERR_INVALID_ARG;

@@ -8,6 +8,7 @@
 #include <climits>
 #include <cstdint>
 
+#include "ps_nvtx.h"
 #include "internal.h"
 #include "ps_common.cuh"
 #include "psppo.h"
@@ -342,8 +343,11 @@ __global__ void __launch_bounds__(kFinThreads)
     }
     const double r = exp(lp - static_cast<double>(oldlogp[i]));
     const double A = adv[i], wt = w[i];
-    const double clipped = fmin(fmax(r, 1.0 - eps), 1.0 + eps);
-    const double sur = fmin(r * A, clipped * A);
+    // min and clip as the definition has them: a NaN ratio (a non-finite input or a bad token
+    // id) gives a NaN surrogate, which fmin / fmax alone would replace by the other operand
+    const double clipped = r != r ? r : fmin(fmax(r, 1.0 - eps), 1.0 + eps);
+    const double ra = r * A, ca = clipped * A;
+    const double sur = (ra != ra || ca != ca) ? NAN : fmin(ra, ca);
     rl = -loss_scale * wt * sur;
     const bool bind = (A > 0.0 && r > 1.0 + eps) || (A < 0.0 && r < 1.0 - eps);
     lse[i] = static_cast<float>(l);
@@ -471,6 +475,7 @@ size_t ps_sample_cutoffs_workspace_size(int, int, int) { return kWsHeader; }
 int ps_sample_cutoffs(int P, int K, int T_max, const uint64_t* q, const int32_t* L, uint64_t seed, uint64_t step,
                       int64_t traj_base, int mode, int32_t* H, int32_t* n, float* w_tab, void* ws, size_t ws_bytes,
                       ps_stream_t stream) {
+  NvtxRange nvtx_range("ps_sample_cutoffs");
   if (P < 1 || K < 1 || K > 8192 || T_max < 1 || T_max > (1 << 24) || traj_base < 0) return PS_ERR_INVALID_ARG;
   if (static_cast<int64_t>(P) * K > INT32_MAX) return PS_ERR_INVALID_ARG;
   if (mode != PS_MODE_TRUNC && mode != PS_MODE_FULL && mode != PS_MODE_TRUNC_ZERO) return PS_ERR_INVALID_ARG;
@@ -497,6 +502,7 @@ int ps_pack_prefixes(int P, int K, int T_max, int d, int dtype, const int32_t* L
                      const void* hid_full, int64_t capacity, int32_t* cu_seqlens, int32_t* src_row,
                      int32_t* row_traj, int32_t* row_pos, int32_t* tok, float* oldlogp, float* w, float* adv,
                      void* hid_packed, int64_t* h_num_rows, void* ws, size_t ws_bytes, ps_stream_t stream) {
+  NvtxRange nvtx_range("ps_pack_prefixes");
   if (P < 1 || K < 1 || T_max < 1 || capacity < 0 || !dtype_ok(dtype)) return PS_ERR_INVALID_ARG;
   if (static_cast<int64_t>(P) * K > (1 << 24)) return PS_ERR_INVALID_ARG;
   if (adv_mode != PS_ADV_CENTERED && adv_mode != PS_ADV_GROUP_NORM) return PS_ERR_INVALID_ARG;
@@ -537,6 +543,7 @@ int ps_lmhead_ppo_fwd(int64_t N, int d, int V, int dtype, const void* Hpk, const
                       const float* oldlogp, const float* adv, const float* w, double eps, double loss_scale,
                       double* loss, float* lse, float* logp, float* ratio, float* coef, float* row_loss, void* ws,
                       size_t ws_bytes, ps_stream_t stream) {
+  NvtxRange nvtx_range("ps_lmhead_ppo_fwd");
   if (N < 0 || N > INT32_MAX || V < 1 || !dtype_ok(dtype) || !d_ok(d, dtype)) return PS_ERR_INVALID_ARG;
   if (!(eps >= 0.0) || !loss || (N > 0 && (!Hpk || !W || !tok || !oldlogp || !adv || !w || !lse || !logp ||
                                            !ratio || !coef)))
@@ -581,6 +588,7 @@ size_t ps_lmhead_ppo_bwd_workspace_size(int64_t N, int d, int V, int dtype, int6
 int ps_lmhead_ppo_bwd(int64_t N, int d, int V, int dtype, const void* Hpk, const void* W, const int32_t* tok,
                       const float* lse, const float* coef, float* dH, float* dW, int flags, void* ws,
                       size_t ws_bytes, ps_stream_t stream) {
+  NvtxRange nvtx_range("ps_lmhead_ppo_bwd");
   if (N < 0 || N > INT32_MAX || V < 1 || !dtype_ok(dtype) || !d_ok(d, dtype)) return PS_ERR_INVALID_ARG;
   if (flags != PS_DW_OVERWRITE && flags != PS_DW_ACCUMULATE) return PS_ERR_INVALID_ARG;
   if (N > 0 && (!Hpk || !W || !tok || !lse || !coef)) return PS_ERR_INVALID_ARG;

@@ -80,3 +80,38 @@ def test_capacity_and_bad_token_and_small_workspace():
         B.ps_lmhead_ppo_fwd(up.N, cfg.d, cfg.V, B.PS_DTYPE_BF16, up.hid, D["W"], up.tok, up.oldlogp, up.adv, up.w,
                             0.2, 1.0, up.loss, up.lse, up.logp, up.ratio, up.coef, None, small)
     assert e.value.status == B.PS_ERR_WORKSPACE
+
+
+def test_non_finite_inputs_stay_in_their_rows():
+    # A NaN hidden state poisons its own row, the loss and the dW sum over rows, and nothing else;
+    # an old log-prob of +inf gives ratio 0 and a finite loss. No status bit is set: non-finite
+    # inputs are passed through, not detected.
+    from synthetic import get_config, make_batch
+    from paper_2606_29758_gb300 import PassShape, UpdatePass
+    cfg = get_config("mid")
+    b = make_batch(cfg, device="cuda")
+    D = b.dev
+
+    def run(hid, old):
+        up = UpdatePass(PassShape(cfg.P, cfg.K, b.T_max, cfg.d, cfg.V, b.total_len, torch.bfloat16, 128),
+                        eps=cfg.eps, loss_scale=cfg.loss_scale)
+        up.run(D["q"], D["L"], D["R"], D["tok_full"], old, hid, D["W"], cfg.seed, cfg.step)
+        torch.cuda.synchronize()
+        up.check_status()
+        return up
+
+    clean = run(D["hid_full"], D["oldlogp_full"])
+    N = clean.N
+    hid = D["hid_full"].clone()
+    hid[0, 5] = float("nan")                 # token 1 of completion 0: always packed, as row 0
+    bad = run(hid, D["oldlogp_full"])
+    assert bad.N == N and torch.isnan(bad.lse[0]) and torch.isnan(bad.row_loss[0])
+    assert torch.isnan(bad.loss).all()                 # as in the definition: min and clip keep a NaN
+    for k in ("lse", "logp", "ratio", "coef"):
+        assert torch.equal(getattr(bad, k)[1:N], getattr(clean, k)[1:N]), k
+    assert torch.equal(bad.dH[1:N], clean.dH[1:N]) and torch.isnan(bad.dH[0]).any()
+    old = D["oldlogp_full"].clone()
+    old[0] = float("inf")
+    inf_run = run(D["hid_full"], old)
+    assert float(inf_run.ratio[0]) == 0.0 and torch.isfinite(inf_run.loss).all()
+    assert torch.isfinite(inf_run.dW).all() and torch.isfinite(inf_run.dH[:N]).all()
