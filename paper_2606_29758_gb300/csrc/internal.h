@@ -12,7 +12,8 @@ int device_is_sm103();
 // Forward GEMM with the online-logsumexp epilogue. part: [splits][N] (max2, sum) pairs
 // (max in log2 units); ztok: [N] chosen-token logit.
 int fwd_tile_splits_bf16(int V);   // one partial per 256-column vocabulary tile
-// Vocabulary ranges per row block, at most max_splits (the partials the workspace holds).
+// Vocabulary ranges per row block, at most max_splits (the partials the workspace holds); the
+// score proxy uses the same chooser.
 int choose_fwd_splits_bf16(int64_t N, int d, int V, int num_sms, int max_splits);
 int fwd_gemm_bf16(int64_t N, int d, int V, const void* Hpk, const void* W, const int32_t* tok, float2* part,
                   float* ztok, int splits, uint32_t* status, cudaStream_t s);
@@ -28,7 +29,6 @@ int proxy_gemm_bf16(int64_t N, int d, int V, const void* Hrows, const void* W, c
 // 16): topk [splits][N][16] (logit, column bits).
 int proxy_topk_gemm_bf16(int64_t N, int d, int V, const void* Hrows, const void* W, const int32_t* tok,
                          float4* part, float2* topk, float* ztok, int splits, uint32_t* status, cudaStream_t s);
-// The forward's chooser with at most max_splits contiguous vocabulary ranges (exported for the proxy).
 
 // Backward for one chunk of rows [0, rc) of already offset pointers: recompute dZ into
 // dz ([rc][ldz], operand dtype), then dH = dZ W and dW (+)= dZ^T Hpk.

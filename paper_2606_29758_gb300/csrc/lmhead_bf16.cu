@@ -451,10 +451,10 @@ static int choose_splits(int64_t m_blocks, int64_t n_blocks, int workers, int mi
   return min_splits;
 }
 
-constexpr bool kUsePairs = false;
-// Rows of a K-major B box: each CTA of a pair loads half of the 256-row B tile (16 KB per
-// stage, the size its ring slot holds and its expect-tx counts); a single CTA loads all of it.
-constexpr uint32_t kBRowsBox = kUsePairs ? 128 : kBN;
+// Rows of the K-major B box in the library's GEMMs, which all run one CTA per tile: the whole
+// 256-row B tile. (The CTA-pair kernel, reached only through the GEMM test hook, has each CTA
+// load half of it, 128 rows; see gemm_bf16.)
+constexpr uint32_t kBRowsBox = kBN;
 // Tile height of the forward and of the logit recompute in 128-row halves (see GemmCfg). The
 // forward gains from the wide tile (fewer operand bytes per FLOP) even though its epilogue is
 // then not overlapped; the recompute, whose epilogue also writes dZ, does better with
@@ -490,7 +490,6 @@ int choose_fwd_splits_bf16(int64_t N, int d, int V, int num_sms, int max_splits)
 int fwd_gemm_bf16(int64_t N, int d, int V, const void* Hpk, const void* W, const int32_t* tok, float2* part,
                   float* ztok, int splits, uint32_t* status, cudaStream_t s) {
   CUtensorMap ta, tb;
-  static_assert(!kUsePairs, "the wide forward tile is a single-CTA kernel");
   if (!map_kmajor(&ta, Hpk, N, d, d, kBM * kFwdHalves) || !map_kmajor(&tb, W, V, d, d, kBRowsBox))
     return PS_ERR_INVALID_ARG;
   FwdLseEpi::Params ep{tok, static_cast<int>(N), V, part, ztok};
