@@ -56,7 +56,8 @@ enum { PS_DW_OVERWRITE = 0, PS_DW_ACCUMULATE = 1 };
 /* Device status bits (the word at offset 0 of every workspace). */
 enum {
   PS_DEV_BAD_PMF = 1, PS_DEV_BAD_LENGTH = 2, PS_DEV_CAPACITY = 4,
-  PS_DEV_BAD_TOKEN = 8, PS_DEV_TIMEOUT = 16
+  PS_DEV_BAD_TOKEN = 8, PS_DEV_TIMEOUT = 16,
+  PS_DEV_NONFINITE = 32   /* ps_design_cutoffs: a timestep weight gamma_bar * u is NaN or infinite */
 };
 
 /* Static string for a ps_status value. */
@@ -268,7 +269,8 @@ int ps_reward_uncertainty(int P, int K, int T_max, const int32_t* L, const float
  * an excess over 2^62 from rounding is taken off the largest mass), zero beyond T_p; the
  * deficit 2^62 - sum_h q[p][h-1] is Pr(H = 0): sample with PS_MODE_TRUNC_ZERO. xi [P][T_max]
  * f64 (may be NULL). Inputs: L [B] int32, gamma_full [sum L] f32 in completion order (needed
- * by OPTIMIZED and HEURISTIC, may be NULL otherwise), u [P][T_max] f32 or NULL.
+ * by OPTIMIZED and HEURISTIC, may be NULL otherwise), u [P][T_max] f32 or NULL. A weight
+ * that is NaN or infinite sets PS_DEV_NONFINITE (the design is then undefined).
  * The arithmetic is f64 in the order of the sequential definition (the parallel parts change
  * no rounding), so the masses are reproducible bit for bit.
  * ------------------------------------------------------------------------- */

@@ -199,6 +199,8 @@ def timestep_weights(gamma_bar_p, u_p):
     design keeps xi_t > 0 (Section 3.2 requires xi_T > 0); all-zero weights become all ones."""
     T = len(gamma_bar_p)
     w = [float(gamma_bar_p[t]) * (float(u_p[t]) if u_p is not None else 1.0) for t in range(T)]
+    if not all(math.isfinite(x) for x in w):
+        raise ValueError("non-finite timestep weight: the design is undefined")
     wmax = max(w)
     if not wmax > 0.0:
         return [1.0] * T

@@ -20,7 +20,8 @@ PS_MODE_TRUNC, PS_MODE_FULL, PS_MODE_TRUNC_ZERO = 0, 1, 2
 PS_DTYPE_BF16, PS_DTYPE_F32 = 0, 1
 PS_ADV_CENTERED, PS_ADV_GROUP_NORM = 0, 1
 PS_DW_OVERWRITE, PS_DW_ACCUMULATE = 0, 1
-PS_DEV_BAD_PMF, PS_DEV_BAD_LENGTH, PS_DEV_CAPACITY, PS_DEV_BAD_TOKEN, PS_DEV_TIMEOUT = 1, 2, 4, 8, 16
+PS_DEV_BAD_PMF, PS_DEV_BAD_LENGTH, PS_DEV_CAPACITY, PS_DEV_BAD_TOKEN, PS_DEV_TIMEOUT, PS_DEV_NONFINITE = \
+    1, 2, 4, 8, 16, 32
 
 EXPORTS = [
     "ps_status_string", "ps_version", "ps_workspace_status",
@@ -42,7 +43,7 @@ __all__ = EXPORTS + [
     "PS_ERR_DEVICE_DATA", "PS_ERR_TIMEOUT", "PS_ERR_CUDA", "PS_MODE_TRUNC", "PS_MODE_FULL", "PS_MODE_TRUNC_ZERO",
     "PS_DTYPE_BF16", "PS_DTYPE_F32", "PS_ADV_CENTERED", "PS_ADV_GROUP_NORM", "PS_DW_OVERWRITE",
     "PS_DW_ACCUMULATE", "PS_DEV_BAD_PMF", "PS_DEV_BAD_LENGTH", "PS_DEV_CAPACITY", "PS_DEV_BAD_TOKEN",
-    "PS_DEV_TIMEOUT", "PS_DESIGN_OPTIMIZED", "PS_DESIGN_HEURISTIC", "PS_DESIGN_UNIFORM",
+    "PS_DEV_TIMEOUT", "PS_DEV_NONFINITE", "PS_DESIGN_OPTIMIZED", "PS_DESIGN_HEURISTIC", "PS_DESIGN_UNIFORM",
     "PS_DESIGN_TIME_PRIOR", "PS_DESIGN_FIXED",
 ]
 

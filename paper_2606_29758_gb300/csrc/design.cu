@@ -329,6 +329,7 @@ __global__ void __launch_bounds__(kDesignThreads)
         if (t < L[p * K + j]) acc = __dadd_rn(acc, static_cast<double>(gamma[off[j] + t]));
       double v = __ddiv_rn(acc, static_cast<double>(K));
       if (u) v = __dmul_rn(v, static_cast<double>(u[static_cast<int64_t>(p) * T_max + t]));
+      if (!isfinite(v)) raise_status(status, PS_DEV_NONFINITE);
       w[t] = v;
       wmax = fmax(wmax, v);
     }

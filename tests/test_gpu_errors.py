@@ -115,3 +115,25 @@ def test_non_finite_inputs_stay_in_their_rows():
     inf_run = run(D["hid_full"], old)
     assert float(inf_run.ratio[0]) == 0.0 and torch.isfinite(inf_run.loss).all()
     assert torch.isfinite(inf_run.dW).all() and torch.isfinite(inf_run.dH[:N]).all()
+
+
+def test_non_finite_design_weight_sets_its_bit():
+    B = _B()
+    from synthetic import get_config
+    from synthetic.generate import draw_design_inputs, draw_lengths
+    cfg = get_config("mid")
+    L = draw_lengths(cfg)
+    gamma, u = draw_design_inputs(cfg, L)
+    gamma[3] = np.nan
+    T = int(L.max())
+    q = torch.empty(cfg.P, T, dtype=torch.int64, device="cuda")
+    ws = torch.zeros(B.ps_design_cutoffs_workspace_size(cfg.P, cfg.K, T), dtype=torch.uint8, device="cuda")
+    B.ps_design_cutoffs(cfg.P, cfg.K, T, torch.from_numpy(L).cuda(), torch.from_numpy(gamma).cuda(),
+                        torch.from_numpy(u).cuda(), 40.0, B.PS_DESIGN_OPTIMIZED, 0.0, q, None, ws)
+    rc, bits = B.ps_workspace_status(ws)
+    assert rc == B.PS_ERR_DEVICE_DATA and bits & B.PS_DEV_NONFINITE
+    # the same inputs with the NaN removed are accepted
+    gamma[3] = 1.0
+    B.ps_design_cutoffs(cfg.P, cfg.K, T, torch.from_numpy(L).cuda(), torch.from_numpy(gamma).cuda(),
+                        torch.from_numpy(u).cuda(), 40.0, B.PS_DESIGN_OPTIMIZED, 0.0, q, None, ws)
+    assert B.ps_workspace_status(ws)[0] == B.PS_OK

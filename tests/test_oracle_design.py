@@ -247,3 +247,10 @@ def test_binarized_labels_extremes_and_streams():
     whole = design.binarize_rewards(R, 5, 3)
     assert np.array_equal(design.binarize_rewards(R[7:], 5, 3, traj_base=7), whole[7:])
     assert not np.array_equal(design.binarize_rewards(R, 5, 4), whole)    # the step changes the draw
+
+
+def test_non_finite_weights_are_refused():
+    with pytest.raises(ValueError):
+        design.timestep_weights(np.array([1.0, np.nan, 2.0]), None)
+    with pytest.raises(ValueError):
+        design.timestep_weights(np.array([1.0, 2.0]), np.array([np.inf, 0.1]))
