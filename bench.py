@@ -10,12 +10,13 @@ value: prefix tokens/s, whole job (sum of packed rows over all steps and ranks d
 by the max over ranks of the device-timed region). The credited work of a step is
 6 N d V FLOPs (forward GEMM, dH, dW; the backward's logit recompute is not credited).
 
-    python bench.py [--gpus N] [--steps K] [--warmup W] [--impl ours|reference]
+    python bench.py [--gpus N] [--steps K] [--warmup W] [--impl ours|reference|torch]
 
 With --gpus N > 1 (launched by torchrun) every rank runs its own replica of the
 workload on its own GPU: the pass has no cross-rank exchange in this form
 (weak scaling). --impl reference times the CPU float64 oracle on bounded samples of
-the same workload, on the host cores.
+the same workload, on the host cores. --impl torch (context only) runs the head of the same step
+in eager PyTorch with materialised logits.
 """
 from __future__ import annotations
 
@@ -208,7 +209,8 @@ def run_ours(args):
                   "zero_advantage_fraction": float((adv_last == 0).float().mean().item()),
                   "pack_gbs": 2.0 * float(np.mean(step_rows)) * cfg.d * (2 if cfg.dtype == "bf16" else 4)
                   / (float(per[:, 1].mean()) * 1e-3) / 1e9,
-                  "sample_us": float(per[:, 0].mean()) * 1e3}
+                  "sample_us": float(per[:, 0].mean()) * 1e3,
+                  "peak_device_memory_gb": torch.cuda.max_memory_allocated() / 1e9}
 
     ms_max = ms
     rows_all = rows
@@ -453,12 +455,70 @@ def run_reference(args):
     }))
 
 
+def run_torch(args):
+    """Context arm: the same step with the head in eager PyTorch (cuBLAS GEMMs, logits
+    materialised per row chunk, autograd for dH and dW); sampling and packing through the library."""
+    import torch
+    from paper_2606_29758_gb300 import PassShape, UpdatePass
+    from synthetic import get_config, make_batch
+    world, rank, local = _dist()
+    if rank != 0:
+        return
+    torch.cuda.set_device(local)
+    dev = f"cuda:{local}"
+    cfg = get_config(args.config)
+    b = make_batch(cfg, device=dev)
+    D = b.dev
+    # the library's backward workspace is not used here: keep it at its minimum (128 rows)
+    up = UpdatePass(PassShape(cfg.P, cfg.K, b.T_max, cfg.d, cfg.V, b.total_len, torch.bfloat16, 128),
+                    device=dev, eps=cfg.eps, loss_scale=cfg.loss_scale)
+    W = D["W"].clone().requires_grad_(True)
+    chunk = args.torch_chunk
+
+    def step(i):
+        up.sample(D["q"], D["L"], cfg.seed, i)
+        n = up.pack(D["L"], D["R"], D["tok_full"], D["oldlogp_full"], D["hid_full"])
+        W.grad = None
+        for r0 in range(0, n, chunk):
+            r1 = min(n, r0 + chunk)
+            h = up.hid[r0:r1].detach().requires_grad_(True)
+            z = (h @ W.t()).float()
+            lp = z.gather(1, up.tok[r0:r1, None].long())[:, 0] - torch.logsumexp(z, dim=1)
+            r = torch.exp(lp - up.oldlogp[r0:r1])
+            A = up.adv[r0:r1]
+            sur = torch.minimum(r * A, torch.clamp(r, 1 - cfg.eps, 1 + cfg.eps) * A)
+            (-(cfg.loss_scale * up.w[r0:r1] * sur).sum()).backward()
+            up.dH[r0:r1] = h.grad
+        return n
+
+    for i in range(args.warmup):
+        step(1000 + i)
+    torch.cuda.synchronize()
+    torch.cuda.reset_peak_memory_stats()
+    e0 = torch.cuda.Event(enable_timing=True)
+    e1 = torch.cuda.Event(enable_timing=True)
+    e0.record()
+    rows = sum(step(i) for i in range(args.steps))
+    e1.record()
+    torch.cuda.synchronize()
+    ms = e0.elapsed_time(e1)
+    print(json.dumps({
+        "impl": "torch-eager", "metric": "prefix tokens/s (fused LM-head PS-PPO fwd+bwd, 1xGB300)",
+        "value": rows / (ms * 1e-3), "unit": "tokens/s", "n_gpus": 1, "steps": args.steps, "warmup": args.warmup,
+        "ms_per_step": ms / args.steps, "higher_is_better": True, "dtype": "bf16",
+        "config": {"workload": describe(cfg), "logit_chunk_rows": chunk},
+        "peak_device_memory_gb": torch.cuda.max_memory_allocated() / 1e9,
+        "note": "context only: the head in eager PyTorch (cuBLAS GEMMs, logits materialised per chunk, "
+                "autograd); cutoffs and packing through the library"}))
+
+
 def main():
     ap = argparse.ArgumentParser()
     ap.add_argument("--gpus", type=int, default=1)
     ap.add_argument("--steps", type=int, default=10)
     ap.add_argument("--warmup", type=int, default=3)
-    ap.add_argument("--impl", choices=["ours", "reference"], default="ours")
+    ap.add_argument("--impl", choices=["ours", "reference", "torch"], default="ours")
+    ap.add_argument("--torch-chunk", type=int, default=16384, help="rows per logit chunk of --impl torch")
     ap.add_argument("--config", default=WORKLOAD)
     ap.add_argument("--chunk-rows", type=int, default=65536)
     ap.add_argument("--cpu-rows", type=int, default=256)
@@ -470,6 +530,8 @@ def main():
         args.warmup = 3
     if args.impl == "reference":
         run_reference(args)
+    elif args.impl == "torch":
+        run_torch(args)
     else:
         run_ours(args)
 
