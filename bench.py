@@ -322,7 +322,8 @@ def run_ours(args):
         "config": {"workload": describe(cfg),
                    "global_batch": cfg.B * world, "mean_prefix_rows": mean_rows, "sum_lengths": b.total_len,
                    "bwd_chunk_rows": args.chunk_rows,
-                   "l2": "inputs larger than L2 (hidden states 2.1 GB, W 1.1 GB)",
+                   "l2": f"inputs larger than L2 (hidden states {b.total_len * cfg.d * 2 / 1e9:.1f} GB, "
+                         f"W {cfg.V * cfg.d * 2 / 1e9:.2f} GB, dZ chunk {args.chunk_rows * cfg.V * 2 / 1e9:.1f} GB)",
                    "parallelism": "replicas" if world > 1 else "single GPU"},
         "pct_bf16_peak": {"credited_6NdV_tflops": credited_tf, "frac_of_sustained": credited_tf / peak_tf,
                           "frac_of_burst": credited_tf / peaks["bf16_tflops"],
