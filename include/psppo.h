@@ -228,6 +228,9 @@ int ps_lmhead_score_proxy(int64_t N, int d, int V, int dtype, const void* Hrows,
  * f32 in completion order (as from ps_lmhead_score_proxy). Limits: K <= 64, 1 <= topk <= 16.
  * ------------------------------------------------------------------------- */
 size_t ps_reward_uncertainty_workspace_size(int P, int K);
+int ps_reward_uncertainty(int P, int K, int T_max, const int32_t* L, const float* R, int topk,
+                          const int32_t* top_idx, const float* top_prob, float* u,
+                          void* ws, size_t ws_bytes, ps_stream_t stream);
 
 /* ---------------------------------------------------------------------------
  * ps_binarize_rewards -- binary labels of continuous rewards, for u_t only.
@@ -245,9 +248,6 @@ size_t ps_reward_uncertainty_workspace_size(int P, int K);
  * ------------------------------------------------------------------------- */
 int ps_binarize_rewards(int B, const float* R, uint64_t seed, uint64_t step, int64_t traj_base,
                         float* y, ps_stream_t stream);
-int ps_reward_uncertainty(int P, int K, int T_max, const int32_t* L, const float* R, int topk,
-                          const int32_t* top_idx, const float* top_prob, float* u,
-                          void* ws, size_t ws_bytes, ps_stream_t stream);
 
 /* ---------------------------------------------------------------------------
  * ps_design_cutoffs -- the per-prompt cutoff distribution and its integer masses.
