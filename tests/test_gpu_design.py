@@ -304,3 +304,45 @@ def test_binarized_rewards_bit_exact_and_u_from_them():
     assert np.array_equal(cd.y.cpu().numpy(), labels)
     u_ref = design.reward_uncertainty(L, cfg.K, labels, idx, prob)
     np.testing.assert_allclose(cd.u.cpu().numpy(), u_ref, atol=2e-7)
+
+
+@pytest.mark.parametrize("name", ["7b", "long"])
+def test_proxy_and_top16_at_full_size(name):
+    # the launch configuration of the design stage in the benchmark: every rollout token of the
+    # batch through the head (per-tile schedule without top-k, contiguous ranges with it); sampled
+    # rows against the oracle, which evaluates them one by one
+    from paper_2606_29758_gb300 import CutoffDesign, DesignShape
+    cfg = get_config(name)
+    b = make_batch(cfg, device="cuda")
+    D = b.dev
+    N, k = b.total_len, 16
+    cd = CutoffDesign(DesignShape(cfg.P, cfg.K, b.T_max, cfg.d, cfg.V, N, k))
+    cd.score(D["hid_full"], D["W"], D["tok_full"])
+    g_topk, lp_topk = cd.gamma.clone(), cd.logp.clone()
+    plain = CutoffDesign(DesignShape(cfg.P, cfg.K, b.T_max, cfg.d, cfg.V, N, 0))
+    plain.score(D["hid_full"], D["W"], D["tok_full"])
+    torch.cuda.synchronize()
+    cd.check_status()
+    plain.check_status()
+    rng = np.random.default_rng(17)
+    rows = np.unique(np.concatenate([rng.choice(N, 60, replace=False), [0, N - 1]]))
+    from synthetic.generate import hidden_rows
+    H = widen(cfg, hidden_rows(cfg, rows))
+    W = widen(cfg, b.W)
+    tok = b.tok_full[rows]
+    g_ref, lp_ref = design.score_proxy(H, W, tok)
+    sel = torch.from_numpy(rows).cuda()
+    for g, lp in ((g_topk, lp_topk), (plain.gamma, plain.logp)):
+        np.testing.assert_allclose(g[sel].cpu().numpy(), g_ref, rtol=2e-4)
+        np.testing.assert_allclose(lp[sel].cpu().numpy(), lp_ref, rtol=1e-4, atol=2e-4)
+    gi, gp = cd.top_idx[sel].cpu().numpy(), cd.top_prob[sel].cpu().numpy()
+    z = H @ W.T
+    P = np.exp(z - z.max(axis=1, keepdims=True))
+    P /= P.sum(axis=1, keepdims=True)
+    r = np.arange(len(rows))[:, None]
+    np.testing.assert_allclose(gp, P[r, gi], rtol=2e-4, atol=1e-9)
+    ridx, rprob = design.topk_policy(H, W, k)
+    np.testing.assert_allclose(P[r, gi].sum(axis=1), rprob.sum(axis=1), rtol=1e-5)
+    zk = np.sort(z, axis=1)[:, ::-1]
+    clear = (zk[:, k - 1] - zk[:, k]) > 1e-3
+    assert np.array_equal(np.sort(gi[clear], axis=1), np.sort(ridx[clear], axis=1))
