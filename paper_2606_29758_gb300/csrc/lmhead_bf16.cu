@@ -138,7 +138,7 @@ struct FwdProxyEpi {
 
 // FwdProxyEpi plus the 16 largest logits of the unit's vocabulary range (Appendix I: u_t uses
 // the top 16 next tokens). The list stays sorted (descending, lower column first on ties) in
-// registers; a 32-column slice is scanned only if its maximum beats the current 16th value.
+// registers; only the values of a 32-column slice above the current 16th value are inserted.
 constexpr int kTopK = 16;
 struct FwdProxyTopkEpi {
   struct Params {
@@ -459,8 +459,11 @@ constexpr uint32_t kBRowsBox = kBN;
 // forward gains from the wide tile (fewer operand bytes per FLOP) even though its epilogue is
 // then not overlapped; the recompute, whose epilogue also writes dZ, does better with
 // 128-row tiles and double-buffered accumulators (7B-shaped step, measured back to back).
-constexpr int kFwdHalves = 2;
 constexpr int kRecHalves = 1;
+// The forward's (and score proxy's) tile height depends on the hidden size: its K loop is d long,
+// while the epilogue of a wide tile is a fixed cost that is not overlapped. Measured back to back:
+// at d = 3584 the wide tile is 1% faster, at d = 1536 the 128-row tile is 7% faster.
+static int fwd_halves(int d) { return d < 2560 ? 1 : 2; }
 
 // The forward keeps one band of row blocks in flight; every CTA re-reads its row block for
 // every vocabulary tile, so the band's hidden rows must stay in L2 (129 MB) next to the W
@@ -469,7 +472,7 @@ constexpr int kRecHalves = 1;
 constexpr double kFwdBandL2Bytes = 30e6;
 
 static int fwd_band_max(int d) {
-  const double block_bytes = static_cast<double>(kBM * kFwdHalves) * d * 2.0;
+  const double block_bytes = static_cast<double>(kBM * fwd_halves(d)) * d * 2.0;
   const int b = static_cast<int>(kFwdBandL2Bytes / block_bytes);
   return b < 1 ? 1 : b;
 }
@@ -481,7 +484,7 @@ static int fwd_band_max(int d) {
 int choose_fwd_splits_bf16(int64_t N, int d, int V, int num_sms, int max_splits) {
   const int nb = fwd_tile_splits_bf16(V);
   if (max_splits >= nb) return nb;
-  const int rows = kBM * kFwdHalves;
+  const int rows = kBM * fwd_halves(d);
   int lo = (num_sms + fwd_band_max(d) - 1) / fwd_band_max(d);
   if (lo > max_splits) lo = max_splits;
   return choose_splits((N + rows - 1) / rows, nb, num_sms, lo, max_splits);
@@ -489,13 +492,16 @@ int choose_fwd_splits_bf16(int64_t N, int d, int V, int num_sms, int max_splits)
 
 int fwd_gemm_bf16(int64_t N, int d, int V, const void* Hpk, const void* W, const int32_t* tok, float2* part,
                   float* ztok, int splits, uint32_t* status, cudaStream_t s) {
+  const int halves = fwd_halves(d);
   CUtensorMap ta, tb;
-  if (!map_kmajor(&ta, Hpk, N, d, d, kBM * kFwdHalves) || !map_kmajor(&tb, W, V, d, d, kBRowsBox))
+  if (!map_kmajor(&ta, Hpk, N, d, d, kBM * halves) || !map_kmajor(&tb, W, V, d, d, kBRowsBox))
     return PS_ERR_INVALID_ARG;
   FwdLseEpi::Params ep{tok, static_cast<int>(N), V, part, ztok};
   const int workers = num_sms_current();
   const int band = splits == fwd_tile_splits_bf16(V) ? fwd_band_max(d) : (workers + splits - 1) / splits;
-  return launch_gemm_single<false, false, FwdLseEpi, kFwdHalves>(ta, tb, N, V, d, splits, band, ep, status, s);
+  if (halves == 1)
+    return launch_gemm_single<false, false, FwdLseEpi, 1>(ta, tb, N, V, d, splits, band, ep, status, s);
+  return launch_gemm_single<false, false, FwdLseEpi, 2>(ta, tb, N, V, d, splits, band, ep, status, s);
 }
 
 // Bands (row blocks walked together) of the backward GEMMs. Recompute: 48 row blocks share
@@ -507,13 +513,16 @@ constexpr int kBandGrad = 1;
 
 int proxy_gemm_bf16(int64_t N, int d, int V, const void* Hrows, const void* W, const int32_t* tok, float4* part,
                     float* ztok, int splits, uint32_t* status, cudaStream_t s) {
+  const int halves = fwd_halves(d);
   CUtensorMap ta, tb;
-  if (!map_kmajor(&ta, Hrows, N, d, d, kBM * kFwdHalves) || !map_kmajor(&tb, W, V, d, d, kBRowsBox))
+  if (!map_kmajor(&ta, Hrows, N, d, d, kBM * halves) || !map_kmajor(&tb, W, V, d, d, kBRowsBox))
     return PS_ERR_INVALID_ARG;
   FwdProxyEpi::Params ep{tok, static_cast<int>(N), V, part, ztok};
   const int workers = num_sms_current();
   const int band = splits == fwd_tile_splits_bf16(V) ? fwd_band_max(d) : (workers + splits - 1) / splits;
-  return launch_gemm_single<false, false, FwdProxyEpi, kFwdHalves>(ta, tb, N, V, d, splits, band, ep, status, s);
+  if (halves == 1)
+    return launch_gemm_single<false, false, FwdProxyEpi, 1>(ta, tb, N, V, d, splits, band, ep, status, s);
+  return launch_gemm_single<false, false, FwdProxyEpi, 2>(ta, tb, N, V, d, splits, band, ep, status, s);
 }
 
 int proxy_topk_gemm_bf16(int64_t N, int d, int V, const void* Hrows, const void* W, const int32_t* tok,
