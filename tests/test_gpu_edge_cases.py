@@ -69,3 +69,19 @@ def test_all_cutoffs_zero_gives_an_empty_pass():
     assert np.all(up.cu_seqlens.cpu().numpy() == 0)
     assert up.loss.item() == 0.0
     assert bool((up.dW == 0).all())      # overwritten with zeros, not left as it was
+
+
+@pytest.mark.parametrize("name,over", [
+    # the largest group the sampler takes (K = 8192, its shared-memory scan), short completions
+    ("max_group", dict(P=1, K=8192, len_lo=1, len_hi=4, d=8, V=5)),
+    # a horizon of 2^20 steps (two completions of up to a million tokens), a tiny head
+    ("long_horizon", dict(P=1, K=2, len_lo=1 << 19, len_hi=1 << 20, d=8, V=7)),
+])
+def test_largest_groups_and_horizons_match_oracle(name, over):
+    cfg = replace(_BASE, name=name, **over)
+    b, up = gpu_pass(cfg, chunk_rows=1 << 16)
+    g = to_np(up, up.N)
+    N, pk = check_prefix(cfg, b, g)
+    assert N == up.N and b.T_max == int(b.L.max())
+    stats = check_head(cfg, b, g, pk)
+    print(name, N, b.T_max, stats)
