@@ -74,8 +74,9 @@ def test_all_cutoffs_zero_gives_an_empty_pass():
 @pytest.mark.parametrize("name,over", [
     # the largest group the sampler takes (K = 8192, its shared-memory scan), short completions
     ("max_group", dict(P=1, K=8192, len_lo=1, len_hi=4, d=8, V=5)),
-    # a horizon of 2^20 steps (two completions of up to a million tokens), a tiny head
-    ("long_horizon", dict(P=1, K=2, len_lo=1 << 19, len_hi=1 << 20, d=8, V=7)),
+    # a horizon of 2^20 steps (two completions of up to a million tokens), a tiny head; seed 3
+    # draws different rewards for the two, so the advantages (and gradients) are not zero
+    ("long_horizon", dict(P=1, K=2, len_lo=1 << 19, len_hi=1 << 20, d=8, V=7, seed=3)),
 ])
 def test_largest_groups_and_horizons_match_oracle(name, over):
     cfg = replace(_BASE, name=name, **over)
@@ -85,3 +86,4 @@ def test_largest_groups_and_horizons_match_oracle(name, over):
     assert N == up.N and b.T_max == int(b.L.max())
     stats = check_head(cfg, b, g, pk)
     print(name, N, b.T_max, stats)
+    assert np.any(g["adv"] != 0) and np.abs(g["dW"]).max() > 0
