@@ -2,7 +2,6 @@
 exact enumeration over every cutoff combination, and Monte Carlo over seeds
 with the exact cutoff-induced variance as the tolerance."""
 import itertools
-import math
 
 import numpy as np
 import pytest
