@@ -1,9 +1,13 @@
-"""One PS-PPO LM-head update pass through the C ABI, with buffers held in torch.
+"""The PS-PPO LM-head update pass through the C ABI, with buffers held in torch.
 
 UpdatePass owns the device buffers of one batch shape (allocated once with torch,
 sized for the worst case N = sum L) and runs the four library calls in order on the
 current stream: cutoffs -> packed prefixes -> fused forward -> fused backward.
 The only host synchronisation is reading N after packing.
+CutoffDesign does the same for the cutoff design upstream of the update (score
+proxy and top-k next tokens, u_t, and the design into sampler masses).
+InputStager copies the next batch's inputs from pinned host memory on its own
+stream while the current pass runs.
 """
 from __future__ import annotations
 
