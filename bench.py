@@ -135,7 +135,8 @@ def run_ours(args):
     cfg = get_config(args.config)
     b = make_batch(cfg, device=dev)
     D = b.dev
-    shape = PassShape(cfg.P, cfg.K, b.T_max, cfg.d, cfg.V, b.total_len, torch.bfloat16, args.chunk_rows)
+    tdtype = torch.bfloat16 if cfg.dtype == "bf16" else torch.float32
+    shape = PassShape(cfg.P, cfg.K, b.T_max, cfg.d, cfg.V, b.total_len, tdtype, args.chunk_rows)
     up = UpdatePass(shape, device=dev, eps=cfg.eps, loss_scale=cfg.loss_scale)
     stream = torch.cuda.current_stream()
     seed = cfg.seed
@@ -306,7 +307,12 @@ def run_ours(args):
             return {"error": f"{type(e).__name__}: {e}"}
 
     full_control = optional(full_control_run)
-    design = optional(time_design_stage, cfg, b, dev, stream) if not args.no_design else None
+    if args.no_design:
+        design = None
+    elif cfg.dtype != "bf16":
+        design = {"skipped": "the score proxy of the design stage takes bf16 inputs only"}
+    else:
+        design = optional(time_design_stage, cfg, b, dev, stream)
 
     peaks, src = _peaks()
     d, V = cfg.d, cfg.V
@@ -317,6 +323,19 @@ def run_ours(args):
     achieved_tf = fwd_flops / t_fwd / 1e12
     step_s = ms / args.steps * 1e-3
     credited_tf = 6.0 * mean_rows * d * V / step_s / 1e12
+    if cfg.dtype == "bf16":
+        roofline = {"kernel": "umma_gemm_kernel<K,K,FwdLseEpi> (fused forward; + O(N) finalize)",
+                    "bound": "tensor", "achieved": achieved_tf, "peak": peak_tf, "unit": "TFLOP/s",
+                    "frac": achieved_tf / peak_tf, "traffic": FWD_GEMM_TRAFFIC.get(cfg.name),
+                    "algorithmic_per_launch": f"2*N*d*V = {fwd_flops:.4g} FLOP",
+                    "peak_note": f"bf16_tflops_sustained ({src}); kernel timed inside the step"}
+    else:
+        # f32 runs on the CUDA cores: 152 SMs x 128 FP32 lanes x 2 FLOP per FMA at the maximum clock
+        alu_peak = 152 * 128 * 2 * peaks.get("sm_max_mhz", 2070.0) * 1e6 / 1e12
+        roofline = {"kernel": "simt_gemm (f32 fused forward; + O(N) finalize)", "bound": "alu",
+                    "achieved": achieved_tf, "peak": alu_peak, "unit": "TFLOP/s", "frac": achieved_tf / alu_peak,
+                    "traffic": None, "algorithmic_per_launch": f"2*N*d*V = {fwd_flops:.4g} FLOP",
+                    "peak_note": "FP32 FMA lanes x 2 x maximum SM clock (derived, not measured)"}
     # per step: sampler 1, packing 2, forward 3 (GEMM, finalize, loss reduction), backward 3 per
     # chunk (recompute, dH, dW); the backward splits a step's rows into ceil(N / chunk) chunks
     launches = sum(6 + 3 * (-(-n // args.chunk_rows)) for n in step_rows)
@@ -331,7 +350,7 @@ def run_ours(args):
         "higher_is_better": True,
         "scaling": "weak",
         "vs_baseline": None,
-        "dtype": "bf16",
+        "dtype": cfg.dtype,
         "data": "synthetic (seeded generator; random-init head)",
         "config": {"workload": describe(cfg),
                    "global_batch": cfg.B * world, "mean_prefix_rows": mean_rows, "sum_lengths": b.total_len,
@@ -346,11 +365,7 @@ def run_ours(args):
                         "fwd": float(per[:, 2].mean()), "bwd": float(per[:, 3].mean()),
                         "note": "pack includes its one host synchronisation (reading N)"},
         "pass_stats": pass_stats,
-        "roofline": {"kernel": "umma_gemm_kernel<K,K,FwdLseEpi> (fused forward; + O(N) finalize)",
-                     "bound": "tensor", "achieved": achieved_tf, "peak": peak_tf, "unit": "TFLOP/s",
-                     "frac": achieved_tf / peak_tf, "traffic": FWD_GEMM_TRAFFIC.get(cfg.name),
-                     "algorithmic_per_launch": f"2*N*d*V = {fwd_flops:.4g} FLOP",
-                     "peak_note": f"bf16_tflops_sustained ({src}); kernel timed inside the step"},
+        "roofline": roofline,
         "e2e": {"value": e_rows / (e_ms * 1e-3), "unit": "tokens/s", "h2d_bytes_per_step": h2d,
                 "d2h_bytes_per_step": 8, "ms_per_step": e_ms / args.steps,
                 "h2d_alone_ms": h2d_ms, "h2d_alone_gbs": h2d / (h2d_ms * 1e-3) / 1e9,
