@@ -366,6 +366,12 @@ def run_ours(args):
                         "note": "pack includes its one host synchronisation (reading N)"},
         "pass_stats": pass_stats,
         "roofline": roofline,
+        "roofline_backward": ({"kernels": "recompute + dH + dW GEMMs (executed 6*N*d*V per step)", "bound": "tensor",
+                               "achieved": 6.0 * mean_rows * d * V / (float(per[:, 3].mean()) * 1e-3) / 1e12,
+                               "peak": peak_tf, "unit": "TFLOP/s",
+                               "frac": 6.0 * mean_rows * d * V / (float(per[:, 3].mean()) * 1e-3) / 1e12 / peak_tf,
+                               "traffic": None, "peak_note": "bf16_tflops_sustained"}
+                              if cfg.dtype == "bf16" else None),
         "e2e": {"value": e_rows / (e_ms * 1e-3), "unit": "tokens/s", "h2d_bytes_per_step": h2d,
                 "d2h_bytes_per_step": 8, "ms_per_step": e_ms / args.steps,
                 "h2d_alone_ms": h2d_ms, "h2d_alone_gbs": h2d / (h2d_ms * 1e-3) / 1e9,
