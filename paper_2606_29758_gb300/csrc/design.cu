@@ -600,7 +600,10 @@ int ps_lmhead_score_proxy(int64_t N, int d, int V, int dtype, const void* Hrows,
   uint32_t* status = static_cast<uint32_t*>(ws);
   row_sqnorm_kernel<<<num_sms_current() * 8, 256, 0, s>>>(N, d, 1, Hrows, hn);
   if (cudaGetLastError() != cudaSuccess) return PS_ERR_CUDA;
-  const int splits = choose_fwd_splits_bf16(N, d, V, num_sms_current(), S);
+  // With the top-k lists, as many vocabulary ranges as the workspace holds (up to 16): shorter
+  // ranges keep the CTAs of a band closer together along W (16 ranges measured 4% faster than
+  // the 11 the forward's chooser picks at 7B). Without them, the forward's per-tile schedule.
+  const int splits = topk > 0 ? S : choose_fwd_splits_bf16(N, d, V, num_sms_current(), S);
   int rc = topk > 0 ? proxy_topk_gemm_bf16(N, d, V, Hrows, W, tok, part, tpart, ztok, splits, status, s)
                     : proxy_gemm_bf16(N, d, V, Hrows, W, tok, part, ztok, splits, status, s);
   if (rc != PS_OK) return rc;
