@@ -254,3 +254,87 @@ def test_non_finite_weights_are_refused():
         design.timestep_weights(np.array([1.0, np.nan, 2.0]), None)
     with pytest.raises(ValueError):
         design.timestep_weights(np.array([1.0, 2.0]), np.array([np.inf, 0.1]))
+
+
+# ---------------------------------------------------------------- the whole design step, by hand
+def _two_prompt_batch():
+    """Prompt 0: lengths (4, 2), per-token scores (16, 4, 8, 2) and (16, 4), so gamma_bar =
+    (16, 4, 4, 1) over T_0 = 4 (the short completion adds 0 beyond its end) and sqrt(w) =
+    (4, 2, 2, 1), sum 9. Prompt 1: lengths (2, 1), T_1 = 2 < T_max = 4."""
+    L = np.array([4, 2, 2, 1], dtype=np.int32)
+    gamma_full = np.array([16., 4., 8., 2.,  16., 4.,  5., 3.,  7.])
+    return L, gamma_full
+
+
+def test_design_masses_per_prompt_horizon_and_budget_by_hand():
+    L, g = _two_prompt_batch()
+    # budget 2: prompt 0 takes the closed form 2 (4, 2, 2, 1) / 9 (already non-increasing, below
+    # the cap); prompt 1's budget is min(2, T_1) = 2 = T_1, so xi = (1, 1) and H = L surely
+    q, xi = design.design_cutoff_masses(L, 2, g, None, 2.0, "optimized")
+    np.testing.assert_allclose(xi[0], [8 / 9, 4 / 9, 4 / 9, 2 / 9], rtol=1e-15)
+    assert list(xi[1]) == [1.0, 1.0, 0.0, 0.0]
+    # masses: Pr(H = h) = xi_h - xi_{h+1}; Pr(H = 0) = 1 - xi_1 = 1/9 is the deficit
+    np.testing.assert_allclose(q[0].astype(np.float64) / ONE62, [4 / 9, 0.0, 2 / 9, 2 / 9], rtol=1e-15, atol=0)
+    assert int(q[0, 1]) == 0
+    assert abs((ONE62 - sum(int(x) for x in q[0])) / ONE62 - 1 / 9) < 1e-15
+    assert [int(x) for x in q[1]] == [0, ONE62, 0, 0]          # zero beyond T_1, no deficit
+
+
+def test_design_masses_cap_and_budget_above_the_horizon():
+    L, g = _two_prompt_batch()
+    # budget 3.5: prompt 0's closed form starts at 3.5 * 4 / 9 > 1, so the cap saturates xi_1 and
+    # the suffix (w = 4, 4, 1; sqrt 2, 2, 1, sum 5) gets budget 2.5: (1, 1, 0.5). Prompt 1: the
+    # budget exceeds T_1 = 2 and becomes 2 (a budget above the horizon has no design).
+    q, xi = design.design_cutoff_masses(L, 2, g, None, 3.5, "optimized")
+    np.testing.assert_allclose(xi[0], [1.0, 1.0, 1.0, 0.5], rtol=1e-15)
+    assert list(xi[1]) == [1.0, 1.0, 0.0, 0.0]
+    assert [int(x) for x in q[0]] == [0, 0, ONE62 // 2, ONE62 // 2]
+    assert [int(x) for x in q[1]] == [0, ONE62, 0, 0]
+    with pytest.raises(ValueError):
+        design.capped_monotone_design([1.0, 1.0], 3.5)           # what B in place of min(B, T_p) would do
+
+
+def test_design_masses_use_u_per_prompt():
+    L, g = _two_prompt_batch()
+    # u scales the weights step by step: gamma_bar_0 = (16, 4, 4, 1) times u_0 = (1/4, 1, 1/4, 1)
+    # gives w = (4, 4, 1, 1), sqrt (2, 2, 1, 1), sum 6; budget 2: (2/3, 2/3, 1/3, 1/3)
+    u = np.array([[0.25, 1.0, 0.25, 1.0], [1.0, 1.0, 0.0, 0.0]])
+    _, xi = design.design_cutoff_masses(L, 2, g, u, 2.0, "optimized")
+    np.testing.assert_allclose(xi[0], [2 / 3, 2 / 3, 1 / 3, 1 / 3], rtol=1e-15)
+
+
+def test_design_masses_other_strategies_by_hand():
+    L, g = _two_prompt_batch()
+    q, xi = design.design_cutoff_masses(L, 2, g, None, 2.0, "uniform")
+    np.testing.assert_allclose(xi[0], [1.0, 0.75, 0.5, 0.25], rtol=1e-15)
+    assert [int(x) for x in q[0]] == [ONE62 // 4] * 4
+    assert [int(x) for x in q[1]] == [ONE62 // 2, ONE62 // 2, 0, 0]
+    q, xi = design.design_cutoff_masses(L, 2, g, None, 2.0, "fixed", param=2)
+    assert list(xi[0]) == [1.0, 1.0, 0.0, 0.0] and [int(x) for x in q[0]] == [0, ONE62, 0, 0]
+    assert list(xi[1]) == [1.0, 1.0, 0.0, 0.0]
+    q, xi = design.design_cutoff_masses(L, 2, g, None, 2.0, "heuristic")
+    np.testing.assert_allclose(xi[0], [8 / 9, 4 / 9, 4 / 9, 2 / 9], rtol=1e-15)
+    q, xi = design.design_cutoff_masses(L, 2, g, None, 2.0, "time_prior")
+    assert list(xi[1]) == [1.0, 1.0, 0.0, 0.0]                  # budget = T_1: lambda = 0
+    assert abs(xi[0].sum() - 2.0) < 1e-12 and xi[0][0] == 1.0
+
+
+def test_timestep_weight_floor_and_all_zero_rule():
+    w = design.timestep_weights(np.array([4.0, 0.0, 1.0]), None)
+    assert w == [4.0, 4.0 * design.W_FLOOR, 1.0]
+    w = design.timestep_weights(np.array([2.0, 3.0]), np.array([0.5, 0.0]))
+    assert w == [1.0, design.W_FLOOR]
+    assert design.timestep_weights(np.zeros(3), None) == [1.0, 1.0, 1.0]
+    assert design.timestep_weights(np.array([1.0, 2.0]), np.zeros(2)) == [1.0, 1.0]
+    # a weight already above the floor is kept as it is
+    assert design.timestep_weights(np.array([1.0, 2e-12]), None) == [1.0, 2e-12]
+
+
+def test_heuristic_cap_and_running_minimum_by_hand():
+    # closed form 3.5 (4, 2, 2, 1) / 9 starts above 1: the cap clips xi_1 only (the heuristic does
+    # not hand the clipped mass back, so its total falls below the budget)
+    h = design.heuristic_design(np.array([16.0, 4.0, 4.0, 1.0]), 3.5)
+    np.testing.assert_allclose(h, [1.0, 7 / 9, 7 / 9, 3.5 / 9], rtol=1e-15)
+    # sqrt(w) = (1, 4, 2): closed form (1, 4, 2) / 7, then the running minimum holds 1/7
+    h = design.heuristic_design(np.array([1.0, 16.0, 4.0]), 1.0)
+    np.testing.assert_allclose(h, [1 / 7, 1 / 7, 1 / 7], rtol=1e-15)
