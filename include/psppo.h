@@ -301,9 +301,11 @@ int ps_design_cutoffs(int P, int K, int T_max, const int32_t* L, const float* ga
  *    all ceil(V/256) of them, the fastest schedule, fit up to about 14,000 rows at
  *    V = 152064. For f32, N * ceil(V/64) * 8 bytes must fit. Larger problems return
  *    PS_ERR_UNSUPPORTED and launch nothing.
- *  - Set-up: the first call on each device looks up the array's device address
- *    (cudaGetSymbolAddress) with that device current; make that first call before
- *    any stream capture.
+ *  - Set-up: the first call in each device context looks up the array's device
+ *    address (cudaGetSymbolAddress) with that device current; make that first call
+ *    before any stream capture. The address is kept per context: after
+ *    cudaDeviceReset, or with another context current, the next call looks it up
+ *    again (so that call, too, belongs before any capture).
  *  - Sharing: every call on a device uses the same array, which keeps the last call's
  *    contents. Calls that overlap on the GPU (e.g. on two streams without ordering)
  *    race on it; order them. Each call clears the status word it uses.

@@ -7,6 +7,7 @@
 // taken from a file-scope __device__ array of kStaticScratchBytes, which every GPU that
 // loads the library holds until the process exits. The function allocates nothing: no
 // cudaMalloc, no cudaFree, no allocating library routine.
+#include <cuda.h>
 #include <cuda_runtime.h>
 
 #include <mutex>
@@ -21,21 +22,68 @@ constexpr int kMaxDevices = 64;
 static __device__ __align__(256) unsigned char g_fwd_scratch[kStaticScratchBytes];
 
 std::mutex g_mu;
-void* g_scratch_ptr[kMaxDevices] = {};
 
-// Device address of this device's copy of g_fwd_scratch. In host code the symbol is only a
-// host-side stand-in, so the address must come from cudaGetSymbolAddress, once per device,
-// with that device current.
+// The array's device address in one device context. A context that is destroyed and created
+// again (cudaDeviceReset, then any runtime call) loads the module anew, possibly at another
+// address, so the address is keyed on the context's process-unique id (cuCtxGetId).
+struct ScratchSlot {
+  void* ptr = nullptr;
+  unsigned long long ctx_id = 0;
+};
+ScratchSlot g_slot[kMaxDevices];
+
+typedef CUresult (*CtxGetCurrentFn)(CUcontext*);
+typedef CUresult (*CtxGetIdFn)(CUcontext, unsigned long long*);
+struct CtxFns {
+  CtxGetCurrentFn get_current = nullptr;
+  CtxGetIdFn get_id = nullptr;
+};
+
+// Driver entry points through the runtime (the library does not link libcuda itself).
+const CtxFns& ctx_fns() {
+  static CtxFns f;
+  static std::once_flag once;
+  std::call_once(once, [] {
+    void* p = nullptr;
+    cudaDriverEntryPointQueryResult q;
+    if (cudaGetDriverEntryPointByVersion("cuCtxGetCurrent", &p, 12000, cudaEnableDefault, &q) == cudaSuccess &&
+        q == cudaDriverEntryPointSuccess)
+      f.get_current = reinterpret_cast<CtxGetCurrentFn>(p);
+    p = nullptr;
+    if (cudaGetDriverEntryPointByVersion("cuCtxGetId", &p, 12000, cudaEnableDefault, &q) == cudaSuccess &&
+        q == cudaDriverEntryPointSuccess)
+      f.get_id = reinterpret_cast<CtxGetIdFn>(p);
+  });
+  return f;
+}
+
+// Device address of the current context's copy of g_fwd_scratch. In host code the symbol is only
+// a host-side stand-in, so the address comes from cudaGetSymbolAddress, with the device current,
+// once per device context: on the first call, and again after the context has changed.
 int scratch_for_current_device(void** out) {
   int dev = -1;
   if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= kMaxDevices) return PS_ERR_CUDA;
+  const CtxFns& f = ctx_fns();
+  if (f.get_current == nullptr || f.get_id == nullptr) return PS_ERR_CUDA;
   std::lock_guard<std::mutex> lock(g_mu);
-  if (g_scratch_ptr[dev] == nullptr) {
-    void* p = nullptr;
+  void* p = nullptr;
+  CUcontext ctx = nullptr;
+  if (f.get_current(&ctx) != CUDA_SUCCESS) return PS_ERR_CUDA;
+  if (ctx == nullptr) {
+    // no context is current yet: the runtime creates the device's primary context (and makes it
+    // current) on its first call that needs one, such as this lookup
     if (cudaGetSymbolAddress(&p, g_fwd_scratch) != cudaSuccess || p == nullptr) return PS_ERR_CUDA;
-    g_scratch_ptr[dev] = p;
+    if (f.get_current(&ctx) != CUDA_SUCCESS || ctx == nullptr) return PS_ERR_CUDA;
   }
-  *out = g_scratch_ptr[dev];
+  unsigned long long id = 0;
+  if (f.get_id(ctx, &id) != CUDA_SUCCESS) return PS_ERR_CUDA;
+  ScratchSlot& slot = g_slot[dev];
+  if (slot.ptr == nullptr || slot.ctx_id != id) {
+    if (p == nullptr && (cudaGetSymbolAddress(&p, g_fwd_scratch) != cudaSuccess || p == nullptr)) return PS_ERR_CUDA;
+    slot.ptr = p;
+    slot.ctx_id = id;
+  }
+  *out = slot.ptr;
   return PS_OK;
 }
 

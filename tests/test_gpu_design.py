@@ -45,8 +45,6 @@ def test_design_masses_bit_exact(name, budget, strategy):
         q_ref, xi_ref = design.design_cutoff_masses(L, cfg.K, gamma, uu, budget, strategy, param=64.0)
         assert np.array_equal(xi, xi_ref), np.abs(xi - xi_ref).max()
         assert np.array_equal(q, q_ref)
-        if strategy != "uniform":
-            continue
 
 
 @pytest.mark.parametrize("name,budget", [("mid", 40.0), ("7b", 128.0)])

@@ -60,3 +60,50 @@ def test_noalloc_rejects_problems_larger_than_its_scratch():
         B.ps_lmhead_ppo_fwd_noalloc(6_000_000, 3584, 152064, B.PS_DTYPE_BF16, t, t, t, t, t, t,
                                     0.2, 1.0, t, t, t, t, t, t)
     assert e.value.status == B.PS_ERR_UNSUPPORTED
+
+
+def test_noalloc_bad_token_shows_as_nan_in_its_row_and_the_loss():
+    # No workspace comes back from this call, so its status word cannot be read: a token id
+    # outside [0, V) must show as NaN in that row's outputs and in the loss, and nowhere else.
+    from paper_2606_29758_gb300 import _binding as B
+    cfg, D, up = _prepared("mid")
+    N = up.N
+    bad = N // 3
+    tok = up.tok[:N].clone()
+    tok[bad] = cfg.V
+    out = {k: torch.zeros(N, device="cuda") for k in OUTS}
+    loss = torch.zeros(1, dtype=torch.float64, device="cuda")
+    B.ps_lmhead_ppo_fwd_noalloc(N, cfg.d, cfg.V, up.dcode, up.hid, D["W"], tok, up.oldlogp, up.adv, up.w,
+                                cfg.eps, cfg.loss_scale, loss, out["lse"], out["logp"], out["ratio"],
+                                out["coef"], out["row_loss"])
+    torch.cuda.synchronize()
+    assert torch.isnan(loss).all()
+    for k in ("logp", "ratio", "row_loss"):
+        assert torch.isnan(out[k][bad]), k
+    keep = torch.ones(N, dtype=torch.bool, device="cuda")
+    keep[bad] = False
+    for k in OUTS:
+        assert torch.isfinite(out[k][keep]).all(), k
+        assert torch.equal(out[k][keep], getattr(up, k)[:N][keep]), k   # every other row as before
+
+
+def test_noalloc_with_fewer_vocabulary_partials_than_tiles():
+    # About 25k packed rows of the 7B-shaped head (V = 152064): the static scratch holds fewer than
+    # the ceil(V / 256) partials per row, so the forward runs with contiguous vocabulary ranges.
+    from paper_2606_29758_gb300 import _binding as B
+    cfg, D, up = _prepared("7b_p2")
+    N = up.N
+    assert N * 8 * ((cfg.V + 255) // 256) > (64 << 20)
+    for call in range(2):
+        out = {k: torch.full((N,), float("nan"), device="cuda") for k in OUTS}
+        loss = torch.full((1,), float("nan"), dtype=torch.float64, device="cuda")
+        B.ps_lmhead_ppo_fwd_noalloc(N, cfg.d, cfg.V, up.dcode, up.hid, D["W"], up.tok, up.oldlogp, up.adv, up.w,
+                                    cfg.eps, cfg.loss_scale, loss, out["lse"], out["logp"], out["ratio"],
+                                    out["coef"], out["row_loss"])
+        torch.cuda.synchronize()
+        rel = abs(loss.item() - up.loss.item()) / abs(up.loss.item())
+        assert rel < 1e-3, (call, rel)
+        for k in OUTS:
+            ref = getattr(up, k)[:N]
+            err = (out[k] - ref).abs().max().item()
+            assert err <= 2e-4 * max(1.0, ref.abs().max().item()), (call, k, err)
