@@ -110,6 +110,38 @@ class UpdatePass:
                 raise B.PsppoError(rc, f"{name} (device bits {bits:#x})")
 
 
+@dataclass(frozen=True)
+class PromptShard:
+    """One rank's share of a rollout batch in a data-parallel update: the prompts [p0, p1), their
+    completions [k0, k1) and their rows [o0, o1) of the unpacked batch (completion after
+    completion). Advantages are per group, so a shard holds whole groups; its cutoffs are drawn
+    with traj_base = k0, the global index of its first completion, so every completion gets the
+    draw it gets in the whole batch; its loss uses the global scale 1/(P K); and dW sums over the
+    shards (PS_DW_ACCUMULATE after the first shard on one device, an all-reduce across devices)."""
+    p0: int
+    p1: int
+    k0: int
+    k1: int
+    o0: int
+    o1: int
+
+    @property
+    def prompts(self) -> int:
+        return self.p1 - self.p0
+
+
+def prompt_shard(P: int, K: int, L, world: int, rank: int) -> PromptShard:
+    """Contiguous prompt ranges of sizes as equal as possible; L: the batch's completion lengths
+    (host array, B = P K entries)."""
+    if not (0 <= rank < world) or world > P:
+        raise ValueError("need 0 <= rank < world <= P")
+    p0, p1 = rank * P // world, (rank + 1) * P // world
+    k0, k1 = p0 * K, p1 * K
+    lens = [int(x) for x in L]
+    o0 = sum(lens[:k0])
+    return PromptShard(p0, p1, k0, k1, o0, o0 + sum(lens[k0:k1]))
+
+
 class InputStager:
     """Double-buffered host -> device staging of the unpacked batch inputs.
 

@@ -81,12 +81,54 @@ def maxrel(a, b):
     return float(np.abs(a - b).max() / den) if den > 0 else float(np.abs(a - b).max())
 
 
-def check_head(cfg, b, g, pk, rows=None, grads=True, report=None):
-    """Compare the head outputs with the oracle. rows: subset of packed rows (None = all)."""
-    W = widen(cfg, b.W)
-    H = widen(cfg, pk["hid"])
-    f = lmhead.forward(H, W, pk["tok"], pk["oldlogp"], pk["adv"], pk["w"], cfg.eps, cfg.loss_scale, rows=rows)
-    idx = f["rows"]
+# ----------------------------------------------------------------------------- the launch schedule
+# The library's row schedule, restated so that a parity check can touch every place where a
+# launch changes hands: the backward's chunking (csrc/psppo_api.cu) and the row bands of the
+# forward, recompute and dH/dW GEMMs (csrc/lmhead_bf16.cu).
+FWD_BAND_L2_BYTES = 30e6      # hidden rows of one forward band
+REC_BAND_BLOCKS = 48          # 128-row blocks per recompute band
+GRAD_BAND_ROWS = 4 * 256      # dH / dW bands: 4 tiles of 256 rows
+
+
+def bwd_chunks(N, ws_chunk_rows):
+    """[r0, r1) of every backward chunk: as few as a workspace of ws_chunk_rows holds, of equal
+    size rounded up to 128 rows."""
+    chunk = ws_chunk_rows // 128 * 128
+    nch = -(-N // chunk)
+    chunk = -(-(-(-N // nch)) // 128) * 128
+    chunk = min(chunk, N)
+    return [(r0, min(N, r0 + chunk)) for r0 in range(0, N, chunk)]
+
+
+def schedule_rows(cfg, N, ws_chunk_rows, seed=1234):
+    """One row of every 128-row block (seeded), and the rows on both sides of every forward band
+    edge, backward chunk edge, recompute band edge, dH/dW band edge, plus the last row."""
+    rng = np.random.default_rng(seed)
+    starts = np.arange(0, N, 128)
+    rows = set((starts + rng.integers(0, np.minimum(128, N - starts))).tolist())
+
+    def edge(e):
+        rows.update(r for r in (e - 1, e) if 0 <= r < N)
+
+    tile = 128 * (2 if cfg.d >= 2560 else 1)          # the forward's tile height at this d
+    band = max(1, int(FWD_BAND_L2_BYTES // (tile * cfg.d * 2)))
+    for e in range(0, N, band * tile):
+        edge(e)
+    edge(N - N % tile)                                  # the forward's last (partial) tile
+    edge(N - N % 128)
+    for r0, r1 in bwd_chunks(N, ws_chunk_rows):
+        for e in range(r0, r1, REC_BAND_BLOCKS * 128):
+            edge(e)
+        for e in range(r0, r1, GRAD_BAND_ROWS):
+            edge(e)
+        edge(r1)
+        edge(r1 - (r1 - r0) % 256)                      # last dH tile of the chunk
+    rows.add(N - 1)
+    return np.array(sorted(rows), dtype=np.int64)
+
+
+def compare_forward(cfg, g, f, idx):
+    """GPU per-row forward outputs at rows idx against the oracle's values f (same order)."""
     lse_err = float(np.abs(g["lse"][idx] - f["lse"]).max())
     logp_err = float(np.abs(g["logp"][idx] - f["logp"]).max())
     ratio_err = float((np.abs(g["ratio"][idx] - f["ratio"]) / f["ratio"]).max())
@@ -94,12 +136,24 @@ def check_head(cfg, b, g, pk, rows=None, grads=True, report=None):
     cref = f["coef"][~near]
     coef_err = maxrel(g["coef"][idx][~near], cref) if cref.size else 0.0
     rl_err = maxrel(g["row_loss"][idx], f["row_loss"])
-    stats = dict(lse=lse_err, logp=logp_err, ratio=ratio_err, coef=coef_err, row_loss=rl_err, near_clip=int(near.sum()))
+    stats = dict(rows=int(len(idx)), lse=lse_err, logp=logp_err, ratio=ratio_err, coef=coef_err, row_loss=rl_err,
+                 near_clip=int(near.sum()))
     assert lse_err < 2e-4, stats
     assert logp_err < 2e-4, stats
     assert ratio_err < 2e-4, stats
     assert coef_err < 2e-4, stats
     assert rl_err < 2e-4, stats
+    return stats
+
+
+def check_head(cfg, b, g, pk, rows=None, grads=True, report=None):
+    """Compare the head outputs with the oracle. rows: subset of packed rows (None = all)."""
+    W = widen(cfg, b.W)
+    idx = np.arange(len(pk["tok"])) if rows is None else np.asarray(rows, dtype=np.int64)
+    Hs = widen(cfg, pk["hid"][idx])                    # only the rows the oracle evaluates
+    f = lmhead.forward(Hs, W, pk["tok"][idx], pk["oldlogp"][idx], pk["adv"][idx], pk["w"][idx], cfg.eps,
+                       cfg.loss_scale)
+    stats = compare_forward(cfg, g, f, idx)
     if rows is None:
         rel = abs(g["loss"] - f["loss"]) / max(abs(f["loss"]), 1e-300)
         stats["loss_rel"] = rel
@@ -107,14 +161,11 @@ def check_head(cfg, b, g, pk, rows=None, grads=True, report=None):
     if grads:
         # the oracle's backward uses its own lse and coef
         if rows is None:
-            dH, dW = lmhead.backward(H, W, pk["tok"], f["lse"], f["coef"])
+            dH, dW = lmhead.backward(Hs, W, pk["tok"], f["lse"], f["coef"])
             stats["dH"] = maxrel(g["dH"], dH)
             stats["dW"] = maxrel(g["dW"], dW)
         else:
-            lse_o = np.zeros(len(pk["tok"]))
-            coef_o = np.zeros(len(pk["tok"]))
-            lse_o[idx], coef_o[idx] = f["lse"], f["coef"]     # oracle values; only these rows are read
-            dH, _ = lmhead.backward(H, W, pk["tok"], lse_o, coef_o, dh_rows=idx, dw_vocab=[])
+            dH, _ = lmhead.backward(Hs, W, pk["tok"][idx], f["lse"], f["coef"], dw_vocab=[])
             stats["dH"] = maxrel(g["dH"][idx], dH)
         assert stats["dH"] < GRAD_MAXREL, stats
         if "dW" in stats:
@@ -123,4 +174,3 @@ def check_head(cfg, b, g, pk, rows=None, grads=True, report=None):
         report.update(stats)
         report["oracle_rows"], report["oracle_lse"], report["oracle_coef"] = idx, f["lse"], f["coef"]
     return stats
-

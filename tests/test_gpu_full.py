@@ -1,15 +1,19 @@
 """Parity at the workloads' full sizes, in the launch configuration the benchmark times.
 
 Cutoffs, weights, advantages and every packing index/row are compared bit-for-bit with
-the oracle over the whole batch. The head is compared on sampled rows the oracle can
-evaluate one by one (random rows, the largest weights, and rows where the clip binds):
-lse, logp, ratio, coef, row loss and the dH row. For dW, which sums over every row,
-two properties that hold at any size are checked: sum_v dW[v, :] = 0 (the softmax score
-e_o - p sums to zero over the vocabulary) within the bound set by the bf16 rounding of
-dZ, and loss = sum of row losses. Then dW itself: the backward runs again over all N rows
-of the oracle's packed batch with the oracle's lse and coef on the sampled rows and coef = 0
-on every other row (whose dZ row is then zero), so dW = sum over the sampled rows, which the
-oracle evaluates on every vocabulary row that a sampled row chose plus 512 random ones.
+the oracle over the whole batch. The head: on the 1.5B-shaped batch the oracle evaluates the
+forward of every packed row (lse, logp, ratio, coef, row loss) and the total loss (Eq.
+truncated_update_Ghat), compared element by element and within 1e-3 relative. On the larger
+batches it evaluates a stratified set of rows that touches every 128-row block and both sides
+of every place where the launch schedule changes hands (forward bands, backward chunks,
+recompute and dH/dW bands, the last partial tile), plus every row where the clip binds and the
+largest weights. dH is compared on that set on every batch. For dW, which sums over every row,
+two properties that hold at any size are checked: sum_v dW[v, :] = 0 (the softmax score e_o - p
+sums to zero over the vocabulary) within the bound set by the bf16 rounding of dZ, and
+loss = sum of row losses. Then dW itself: the backward runs again over all N rows of the
+oracle's packed batch with the oracle's lse and coef on the stratified rows and coef = 0 on
+every other row (whose dZ row is then zero), so dW = sum over those rows, which the oracle
+evaluates on every vocabulary row that one of them chose plus 512 random ones.
 """
 import numpy as np
 import pytest
@@ -17,7 +21,8 @@ import torch
 
 from synthetic import get_config, make_batch
 
-from gpu_util import GRAD_MAXREL, check_head, oracle_prefix
+from gpu_util import GRAD_MAXREL, LOSS_RTOL, compare_forward, maxrel, oracle_prefix, schedule_rows
+from oracle_pool import oracle_rows
 
 pytestmark = pytest.mark.gpu
 
@@ -56,23 +61,28 @@ def test_full_size(name):
     hid = up.hid[:N].view(torch.int16).cpu().numpy().view(np.uint16)
     assert np.array_equal(hid, pk["hid"])
 
-    # sampled rows for the head
-    rng = np.random.default_rng(1234)
-    coef = _pull(up.coef, N)
-    adv = pk["adv"]
-    bind = np.nonzero((coef == 0) & (adv != 0))[0]
+    # rows for the head: the stratified set, every clip-bound row and the 16 largest weights
+    g = {"lse": _pull(up.lse, N), "logp": _pull(up.logp, N), "ratio": _pull(up.ratio, N), "coef": _pull(up.coef, N),
+         "row_loss": _pull(up.row_loss, N)}
+    bind = np.nonzero((g["coef"] == 0) & (pk["adv"] != 0))[0]
     heavy = np.argsort(pk["w"])[-16:]
-    rows = np.unique(np.concatenate([rng.choice(N, size=min(N, 768), replace=False), heavy,
-                                     bind[:64], [0, N - 1]])).astype(np.int64)
-    g = {"lse": _pull(up.lse, N), "logp": _pull(up.logp, N), "ratio": _pull(up.ratio, N), "coef": coef,
-         "row_loss": _pull(up.row_loss, N), "w": _pull(up.w, N)}
-    dH = np.zeros((N, cfg.d), dtype=np.float32)
-    sel = torch.from_numpy(rows).cuda()
-    dH[rows] = up.dH[sel].cpu().numpy()
-    g["dH"] = dH
-    rep = {}
-    stats = check_head(cfg, b, g, pk, rows=rows, report=rep)
-    print(name, N, len(rows), stats)
+    rows = np.unique(np.concatenate([schedule_rows(cfg, N, CHUNK), bind, heavy])).astype(np.int64)
+    assert np.unique(rows // 128).size == -(-N // 128)          # every 128-row block is touched
+    every_row = name == "1.5b"
+    fwd_rows = np.arange(N) if every_row else rows
+    res = oracle_rows(cfg, b.W, pk["hid"][fwd_rows], pk["tok"][fwd_rows], pk["oldlogp"][fwd_rows],
+                      pk["adv"][fwd_rows], pk["w"][fwd_rows], dh_mask=np.isin(fwd_rows, rows))
+    stats = compare_forward(cfg, g, res, fwd_rows)
+    if every_row:
+        loss_rel = abs(up.loss.item() - res["loss"]) / abs(res["loss"])
+        stats["loss_rel"] = loss_rel
+        assert loss_rel < LOSS_RTOL, stats
+    g_dH = up.dH[torch.from_numpy(rows).cuda()].double().cpu().numpy()
+    stats["dH"] = maxrel(g_dH, res["dH"])
+    print(name, N, "head rows", len(fwd_rows), "dH rows", len(rows), stats)
+    assert stats["dH"] < GRAD_MAXREL, stats
+    at = np.searchsorted(fwd_rows, rows)                        # the stratified rows inside fwd_rows
+    rep = {"oracle_rows": rows, "oracle_lse": res["lse"][at], "oracle_coef": res["coef"][at]}
 
     # loss = sum of row losses (the row losses are checked above)
     total = float(up.row_loss[:N].double().sum().item())
@@ -87,7 +97,7 @@ def test_full_size(name):
     assert ratio < 1.0, ratio
     assert torch.isfinite(up.dW).all() and torch.isfinite(up.dH[:N]).all()
 
-    # dW at full size: same N, chunking and kernels; only the sampled rows carry a coefficient
+    # dW at full size: same N, chunking and kernels; only the stratified rows carry a coefficient
     from oracle import lmhead
     from oracle.pipeline import widen
     from paper_2606_29758_gb300 import _binding as B
@@ -104,6 +114,7 @@ def test_full_size(name):
                         torch.from_numpy(coef32).cuda(), dH2, dW2, B.PS_DW_OVERWRITE, up.ws_bwd)
     torch.cuda.synchronize()
     up.check_status()
+    rng = np.random.default_rng(1234)
     vocab = np.unique(np.concatenate([pk["tok"][idx], rng.choice(cfg.V, size=512, replace=False)]))
     _, dW_ref = lmhead.backward(widen(cfg, pk["hid"][idx]), widen(cfg, b.W), pk["tok"][idx],
                                 lse32[idx].astype(np.float64), coef32[idx].astype(np.float64),
@@ -112,7 +123,7 @@ def test_full_size(name):
     err = float(np.abs(got - dW_ref).max() / np.abs(dW_ref).max())
     print(name, "dW over", len(idx), "rows,", len(vocab), "vocab rows: max-rel", err)
     assert err < GRAD_MAXREL, err
-    # every other row's dZ is zero, so the unsampled rows of dH vanish
+    # every other row's dZ is zero, so the other rows of dH vanish
     others = torch.ones(N, dtype=torch.bool, device="cuda")
     others[torch.from_numpy(idx).cuda()] = False
     assert float(dH2[others].abs().max().item()) == 0.0
