@@ -211,6 +211,10 @@ def run_ours(args):
                   "pack_gbs": 2.0 * float(np.mean(step_rows)) * cfg.d * (2 if cfg.dtype == "bf16" else 4)
                   / (float(per[:, 1].mean()) * 1e-3) / 1e9,
                   "sample_us": float(per[:, 0].mean()) * 1e3,
+                  # algorithmic bytes of one sampler call: the masses q (8 B) read and the weight table
+                  # (4 B) written per (prompt, step), lengths read and (H, n) written per completion
+                  "sample_gbs": (12.0 * cfg.P * b.T_max + 12.0 * cfg.B) / (float(per[:, 0].mean()) * 1e-3) / 1e9,
+                  "sample_bytes": 12 * cfg.P * b.T_max + 12 * cfg.B,
                   "peak_device_memory_gb": torch.cuda.max_memory_allocated() / 1e9}
 
     ms_max = ms
@@ -323,6 +327,13 @@ def run_ours(args):
     achieved_tf = fwd_flops / t_fwd / 1e12
     step_s = ms / args.steps * 1e-3
     credited_tf = 6.0 * mean_rows * d * V / step_s / 1e12
+    # the tensor cores' dense bf16 rate from unit counts and clocks: every SM completes 8192 bf16
+    # FLOP per clock (one 128 x 256 x 16 tcgen05 MMA per 128 clocks), at the median SM clock
+    # sampled during the timed region and at the maximum clock
+    sms = torch.cuda.get_device_properties(dev).multi_processor_count
+    arch_per_mhz = sms * 8192 * 1e6 / 1e12
+    mhz_run = clk.get("sm_mhz") or None
+    mhz_max = clk.get("sm_max_mhz") or peaks.get("sm_max_mhz", 2070.0)
     if cfg.dtype == "bf16":
         roofline = {"kernel": "umma_gemm_kernel<K,K,FwdLseEpi> (fused forward; + O(N) finalize)",
                     "bound": "tensor", "achieved": achieved_tf, "peak": peak_tf, "unit": "TFLOP/s",
@@ -358,9 +369,21 @@ def run_ours(args):
                    "l2": f"inputs larger than L2 (hidden states {b.total_len * cfg.d * 2 / 1e9:.1f} GB, "
                          f"W {cfg.V * cfg.d * 2 / 1e9:.2f} GB, dZ chunk {args.chunk_rows * cfg.V * 2 / 1e9:.1f} GB)",
                    "parallelism": "replicas" if world > 1 else "single GPU"},
-        "pct_bf16_peak": {"credited_6NdV_tflops": credited_tf, "frac_of_sustained": credited_tf / peak_tf,
-                          "frac_of_burst": credited_tf / peaks["bf16_tflops"],
-                          "executed_8NdV_tflops": credited_tf * 8 / 6, "peak_source": src},
+        "pct_bf16_peak": {"credited_6NdV_tflops": credited_tf,
+                          "of_measured_cublas_sustained": credited_tf / peak_tf,
+                          "of_measured_cublas_burst": credited_tf / peaks["bf16_tflops"],
+                          "measured_source": src,
+                          "arch_tflops_at_run_clock": arch_per_mhz * mhz_run if mhz_run else None,
+                          "of_arch_at_run_clock": credited_tf / (arch_per_mhz * mhz_run) if mhz_run else None,
+                          "arch_tflops_at_max_clock": arch_per_mhz * mhz_max,
+                          "of_arch_at_max_clock": credited_tf / (arch_per_mhz * mhz_max),
+                          "of_nominal_2250": credited_tf / 2250.0,
+                          "executed_8NdV_tflops": credited_tf * 8 / 6,
+                          "executed_of_arch_at_run_clock": (credited_tf * 8 / 6) / (arch_per_mhz * mhz_run)
+                          if mhz_run else None,
+                          "arch_note": f"{sms} SMs x 8192 dense bf16 FLOP per SM per clock x SM clock (run: median "
+                                       f"sampled under load; max: the clock limit); nominal 2250 TFLOP/s dense; "
+                                       f"'measured_cublas' = MEASURED_PEAKS.json (torch.matmul 8192^3)"},
         "per_call_ms": {"sample": float(per[:, 0].mean()), "pack": float(per[:, 1].mean()),
                         "fwd": float(per[:, 2].mean()), "bwd": float(per[:, 3].mean()),
                         "note": "pack includes its one host synchronisation (reading N)"},
@@ -383,12 +406,7 @@ def run_ours(args):
     if design is not None:
         out["design_stage"] = design
     if rank == 0 and not args.no_cpu_baseline:
-        cb = optional(cpu_baseline, cfg, b, args.cpu_rows)
-        if "value" in cb:
-            # linear extrapolation from the sample to a whole step of mean_rows packed rows
-            cb["extrapolated_step_s"] = mean_rows / cb["value"]
-            cb["extrapolated_note"] = "extrapolated linearly from the sample to one step's packed rows"
-        out["cpu_baseline"] = cb
+        out["cpu_baseline"] = optional(cpu_baseline, cfg, b, args.cpu_rows)
     if world > 1:
         dist.destroy_process_group()
     if rank == 0:
@@ -405,7 +423,7 @@ def time_design_stage(cfg, b, dev, stream, reps=3):
     D = b.dev
     N = b.total_len
     cd = CutoffDesign(DesignShape(cfg.P, cfg.K, b.T_max, cfg.d, cfg.V, N, 16), device=dev)
-    ev = [torch.cuda.Event(enable_timing=True) for _ in range(4)]
+    ev = [torch.cuda.Event(enable_timing=True) for _ in range(5)]
     t = []
     for r in range(reps + 1):
         ev[0].record(stream)
@@ -415,43 +433,75 @@ def time_design_stage(cfg, b, dev, stream, reps=3):
         ev[2].record(stream)
         cd.design(D["L"], 128.0)
         ev[3].record(stream)
+        cd.design(D["L"], 2048.0)
+        ev[4].record(stream)
         torch.cuda.synchronize()
         if r > 0:
-            t.append([ev[i].elapsed_time(ev[i + 1]) for i in range(3)])
+            t.append([ev[i].elapsed_time(ev[i + 1]) for i in range(4)])
     cd.check_status()
-    pm, um, dm = (float(x) for x in np.mean(np.array(t), axis=0))
-    return {"rows": N, "proxy_topk_ms": pm, "uncertainty_ms": um, "design_ms": dm,
+    saturated = int((cd.xi == 1.0).sum().item())
+    pm, um, dm, dm2 = (float(x) for x in np.mean(np.array(t), axis=0))
+    return {"rows": N, "proxy_topk_ms": pm, "uncertainty_ms": um, "design_ms": dm, "design_ms_budget_2048": dm2,
+            "saturated_steps_budget_2048": saturated,
             "proxy_tflops": 2.0 * N * cfg.d * cfg.V / (pm * 1e-3) / 1e12,
             "note": "score proxy + top-16 over every rollout token (one head GEMM + epilogue), u_t, and the "
-                    "optimized design (budget 128) per prompt; not part of the timed step"}
+                    "optimized design (budget 128, and 2048, where the cap saturates long prefixes) per "
+                    "prompt; not part of the timed step"}
 
 
-def _oracle_sample_pass(cfg, b, W64, rows_in_sample, step):
-    """The oracle, as it stands, on a bounded sample: cutoffs, advantages and packing indices
-    for the whole batch, then the head forward and backward over the first packed rows."""
-    from oracle import lmhead
+def _oracle_prefix(cfg, b, step):
+    """The oracle's cutoffs, advantages and packing indices for the whole batch (one step)."""
     from oracle.cutoffs import sample_cutoffs
     from oracle.pack import group_advantages, pack_prefixes
-    from oracle.pipeline import widen
     H, n, w_tab = sample_cutoffs(b.q, b.L, cfg.K, cfg.seed, step)
     A = group_advantages(b.R, cfg.K, cfg.adv_mode)
-    pk = pack_prefixes(b.L, n, cfg.K, w_tab, A, b.tok_full, b.oldlogp_full, None)
-    s = np.arange(min(rows_in_sample, pk["N"]))
+    return pack_prefixes(b.L, n, cfg.K, w_tab, A, b.tok_full, b.oldlogp_full, None)
+
+
+def _oracle_head(cfg, b, W64, pk, rows):
+    """The oracle's head forward, dH and dW over the first `rows` packed rows of a step."""
+    from oracle import lmhead
+    from oracle.pipeline import widen
+    s = np.arange(min(rows, pk["N"]))
     Hs = widen(cfg, b.hid_full[pk["src_row"][s]])
     f = lmhead.forward(Hs, W64, pk["tok"][s], pk["oldlogp"][s], pk["adv"][s], pk["w"][s], cfg.eps, cfg.loss_scale)
     lmhead.backward(Hs, W64, pk["tok"][s], f["lse"], f["coef"])
     return s.size
 
 
+def _oracle_timing(cfg, b, W64, rows, step):
+    """One step of the oracle, timed in two parts: the whole batch's cutoffs, advantages and packing
+    indices (in full), and the head over a sample of `rows` packed rows. The head's work is linear in
+    the rows (each row's forward and dH; dW sums row by row), so a whole step's time is the prefix
+    time plus N times the head's per-row time."""
+    t0 = time.perf_counter()
+    pk = _oracle_prefix(cfg, b, step)
+    t1 = time.perf_counter()
+    done = _oracle_head(cfg, b, W64, pk, rows)
+    t2 = time.perf_counter()
+    return {"N": pk["N"], "prefix_s": t1 - t0, "head_rows": done, "head_s": t2 - t1}
+
+
+def _oracle_summary(ts):
+    N = float(np.mean([t["N"] for t in ts]))
+    prefix_s = float(np.mean([t["prefix_s"] for t in ts]))
+    head_rate = sum(t["head_rows"] for t in ts) / sum(t["head_s"] for t in ts)
+    step_s = prefix_s + N / head_rate
+    return {"value": N / step_s, "unit": "tokens/s", "head_rows_per_s": head_rate, "prefix_s_per_step": prefix_s,
+            "extrapolated_step_s": step_s, "mean_prefix_rows": N}
+
+
 def cpu_baseline(cfg, b, rows):
     from oracle.pipeline import widen
     W64 = widen(cfg, b.W)
-    t0 = time.perf_counter()
-    done = _oracle_sample_pass(cfg, b, W64, rows, 0)
-    dt = time.perf_counter() - t0
-    return {"value": done / dt, "unit": "tokens/s", "cores": os.cpu_count(), "kind": "oracle",
-            "sample": f"{done} packed rows of one {cfg.name} batch (cutoffs, advantages and packing of the "
-                      f"whole batch; f64 head forward + dH + dW over the sampled rows), {dt:.1f} s"}
+    t = _oracle_timing(cfg, b, W64, rows, 0)
+    out = _oracle_summary([t])
+    out.update({"cores": os.cpu_count(), "kind": "oracle",
+                "sample": f"one {cfg.name} step: cutoffs, advantages and packing indices of the whole batch "
+                          f"({t['prefix_s']:.2f} s), then the f64 head forward + dH + dW over {t['head_rows']} "
+                          f"packed rows ({t['head_s']:.1f} s); value = the step's packed rows / (prefix time + "
+                          f"rows x per-row head time), extrapolated"})
+    return out
 
 
 def run_reference(args):
@@ -471,23 +521,24 @@ def run_reference(args):
     b = make_batch(cfg, device=dev)   # the old log-probs need the full head; on the GPU when present
     W64 = widen(cfg, b.W)
     for i in range(args.warmup):
-        _oracle_sample_pass(cfg, b, W64, args.ref_rows, 1000 + i)
+        _oracle_timing(cfg, b, W64, args.ref_rows, 1000 + i)
     t0 = time.perf_counter()
-    rows = 0
-    for i in range(args.steps):
-        rows += _oracle_sample_pass(cfg, b, W64, args.ref_rows, i)
+    ts = [_oracle_timing(cfg, b, W64, args.ref_rows, i) for i in range(args.steps)]
     dt = time.perf_counter() - t0
-    v = rows / dt
+    summ = _oracle_summary(ts)
+    v = summ["value"]
     print(json.dumps({
         "impl": "reference", "metric": "prefix tokens/s (fused LM-head PS-PPO fwd+bwd, 1xGB300)",
         "value": v, "unit": "tokens/s", "n_gpus": world, "steps": args.steps, "warmup": args.warmup,
-        "ms_per_step": dt / args.steps * 1e3, "higher_is_better": True, "scaling": "weak", "vs_baseline": None,
-        "dtype": "f64", "data": "synthetic (seeded generator; random-init head)",
-        "config": {"workload": describe(cfg),
-                   "sample_rows_per_step": args.ref_rows},
+        "ms_per_step": summ["extrapolated_step_s"] * 1e3, "higher_is_better": True, "scaling": "weak",
+        "vs_baseline": None, "dtype": "f64", "data": "synthetic (seeded generator; random-init head)",
+        "config": {"workload": describe(cfg), "sample_rows_per_step": args.ref_rows},
         "cpu_baseline": {"value": v, "unit": "tokens/s", "cores": os.cpu_count(), "kind": "oracle",
-                         "sample": f"{args.ref_rows} packed rows per step (f64 forward + dH + dW) after "
-                                   f"cutoffs/packing of the whole batch"},
+                         "head_rows_per_s": summ["head_rows_per_s"], "prefix_s_per_step": summ["prefix_s_per_step"],
+                         "sample": f"{args.steps} steps, each: cutoffs, advantages and packing indices of the "
+                                   f"whole batch in full, then the f64 head forward + dH + dW over "
+                                   f"{args.ref_rows} packed rows ({dt:.1f} s in all); value and ms_per_step = "
+                                   f"one whole step extrapolated: prefix time + N x per-row head time"},
         "e2e": {"value": v, "unit": "tokens/s", "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
     }))
 

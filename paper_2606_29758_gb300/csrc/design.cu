@@ -238,34 +238,40 @@ __device__ __forceinline__ bool pav_violates(double Wp, int np, double Wc, int n
 // Pool adjacent violators over w[0..T) (Appendix F) into one lane's stack (element m of the stack
 // at index m * kCapLanes): a new block is merged with the one below it while the block below has
 // the smaller score sqrt(W / n); merged weights add as W_prev + W_last, in the order of the
-// sequential definition, so every block sum is the same double. Returns the number of blocks.
-__device__ int pav_stack_dev(const double* w, int T, double* bW, int32_t* bn) {
+// sequential definition, so every block sum is the same double. Returns the number of blocks (-1
+// if *stop was set before the end).
+__device__ int pav_stack_dev(const double* w, int T, double* bW, int32_t* bn, const volatile int* stop = nullptr) {
   // The top block stays in registers (Wt, nt); the blocks below it are in memory at [0, nb - 1).
   // Memory is read only when a merge uncovers the block below.
   int nb = 0;
   double Wt = 0.0;
   int nt = 0;
   double wnext = T > 0 ? w[0] : 0.0;
-  for (int t = 0; t < T; ++t) {
-    double Wc = wnext;
-    if (t + 1 < T) wnext = w[t + 1];
-    int nc = 1;
-    while (nb > 0 && pav_violates(Wt, nt, Wc, nc)) {
-      Wc = __dadd_rn(Wt, Wc);
-      nc += nt;
-      --nb;
-      if (nb > 0) {
-        Wt = bW[(nb - 1) * kCapLanes];
-        nt = bn[(nb - 1) * kCapLanes];
+  for (int t0 = 0; t0 < T; t0 += 64) {
+    if (stop != nullptr && *stop) return -1;   // abandoned: the caller needs no answer
+    const int t1 = min(T, t0 + 64);
+    for (int t = t0; t < t1; ++t) {
+      if (t + 16 < T) asm volatile("prefetch.global.L1 [%0];" ::"l"(w + t + 16));
+      double Wc = wnext;
+      if (t + 1 < T) wnext = w[t + 1];
+      int nc = 1;
+      while (nb > 0 && pav_violates(Wt, nt, Wc, nc)) {
+        Wc = __dadd_rn(Wt, Wc);
+        nc += nt;
+        --nb;
+        if (nb > 0) {
+          Wt = bW[(nb - 1) * kCapLanes];
+          nt = bn[(nb - 1) * kCapLanes];
+        }
       }
+      if (nb > 0) {
+        bW[(nb - 1) * kCapLanes] = Wt;
+        bn[(nb - 1) * kCapLanes] = nt;
+      }
+      Wt = Wc;
+      nt = nc;
+      ++nb;
     }
-    if (nb > 0) {
-      bW[(nb - 1) * kCapLanes] = Wt;
-      bn[(nb - 1) * kCapLanes] = nt;
-    }
-    Wt = Wc;
-    nt = nc;
-    ++nb;
   }
   if (nb > 0) {
     bW[(nb - 1) * kCapLanes] = Wt;
@@ -274,9 +280,103 @@ __device__ int pav_stack_dev(const double* w, int T, double* bW, int32_t* bn) {
   return nb;
 }
 
+// ---------------------------------------------------------------- capped design: locating the prefix
+// The capped design saturates the smallest prefix s whose suffix design (w[s..T), budget B - s)
+// starts at or below 1. Whether a prefix qualifies is not monotone in s, so it cannot be bisected;
+// instead one pass of pooling from the right gives every suffix's first value at once: once w[t]
+// has been pushed (and pooled with the blocks to its right while it violates the order), the stack
+// holds the pooled blocks of the suffix w[t..T), because the pooled solution of a suffix is unique
+// whatever order its violators are pooled in (only the rounding of the block sums depends on it).
+// With D(t) = sum over those blocks of n_m s_m = sqrt(n_m W_m), the suffix design starts at
+// g(t) = (B - t) s_front / D(t). The pass records whether g(t) is clearly above 1 (0), clearly
+// below (2) or within kCapBand of 1 (1); only the last kind, and the first clear one, are then
+// decided by the exact rounded sequence of the definition.
+constexpr double kCapBand = 0x1p-16;
+constexpr int kMaxNearCap = 64;        // prefixes within the band decided exactly (beyond: the full scan)
+constexpr int kCapStackSmem = 8192;    // stack entries of the status pass held in shared memory
+
+// Float-float numbers (an unevaluated sum hi + lo of two floats, about 44 significant bits): the
+// status pass's block sums and D. Knuth's TwoSum and the Dekker renormalisation.
+struct FF {
+  float hi, lo;
+};
+__device__ __forceinline__ FF ff_add(FF a, FF b) {
+  const float s = a.hi + b.hi;
+  const float bb = s - a.hi;
+  const float e = (a.hi - (s - bb)) + (b.hi - bb) + a.lo + b.lo;
+  const float h = s + e;
+  return FF{h, e - (h - s)};
+}
+
+// One thread: status[t] for t = T-1 down to 0 (see above), in float arithmetic (the FP64 units are
+// far slower). ws[t] = w[t] / max_t w[t] as floats (g does not depend on the scale, and every
+// n W then lies in [1e-12, T]); block sums and D as float-float numbers, roots and the comparison
+// in float: g is within about 2e-7 relative of its exact value, far inside kCapBand. The stack keeps
+// its front block in registers, the next kCapStackSmem entries in shared memory (W, n and the
+// root r = sqrt(n W) of each block, so that a pooled block leaves D as it entered) and deeper ones
+// in gW / gn / gr with stride kCapLanes. Stops early once *stop is set.
+__device__ void cap_status_pass(const float* __restrict__ ws, int T, double B, float2* sW, int32_t* sn, float* sr,
+                                double* gW, int32_t* gn, double* gr, float* status, const volatile int* stop) {
+  int nb = 0;            // blocks below the front
+  FF Wf{0.f, 0.f};       // front block
+  int nf = 0;
+  float rf = 0.f;
+  FF D{0.f, 0.f};
+  const float hi_band = static_cast<float>(1.0 + kCapBand), lo_band = static_cast<float>(1.0 - kCapBand);
+  for (int t = T - 1; t >= 0; --t) {
+    if ((t & 255) == 0 && *stop) return;   // the prefix s = 0 already qualifies: no status is needed
+    if (t >= 32) asm volatile("prefetch.global.L1 [%0];" ::"l"(ws + t - 32));
+    FF Wc{ws[t], 0.f};
+    int nc = 1;
+    // the new block sits left of the front: pool while its mean is below the front's
+    while (nf > 0 && Wf.hi * static_cast<float>(nc) > Wc.hi * static_cast<float>(nf)) {
+      D = ff_add(D, FF{-rf, 0.f});
+      Wc = ff_add(Wc, Wf);
+      nc += nf;
+      if (nb > 0) {
+        --nb;
+        if (nb < kCapStackSmem) {
+          const float2 v = sW[nb];
+          Wf = FF{v.x, v.y};
+          nf = sn[nb];
+          rf = sr[nb];
+        } else {
+          const float2 v = reinterpret_cast<const float2*>(gW)[static_cast<int64_t>(nb) * kCapLanes];
+          Wf = FF{v.x, v.y};
+          nf = gn[static_cast<int64_t>(nb) * kCapLanes];
+          rf = static_cast<float>(gr[static_cast<int64_t>(nb) * kCapLanes]);
+        }
+      } else {
+        nf = 0;
+      }
+    }
+    if (nf > 0) {
+      if (nb < kCapStackSmem) {
+        sW[nb] = make_float2(Wf.hi, Wf.lo);
+        sn[nb] = nf;
+        sr[nb] = rf;
+      } else {
+        reinterpret_cast<float2*>(gW)[static_cast<int64_t>(nb) * kCapLanes] = make_float2(Wf.hi, Wf.lo);
+        gn[static_cast<int64_t>(nb) * kCapLanes] = nf;
+        gr[static_cast<int64_t>(nb) * kCapLanes] = rf;
+      }
+      ++nb;
+    }
+    Wf = Wc;
+    nf = nc;
+    rf = sqrtf(static_cast<float>(nc) * Wc.hi);
+    D = ff_add(D, FF{rf, 0.f});
+    const float num = static_cast<float>(B - static_cast<double>(t)) * rf, den = D.hi * static_cast<float>(nc);
+    status[t] = num > hi_band * den ? 0.f : (num < lo_band * den ? 2.f : 1.f);
+  }
+}
+
+constexpr size_t kDesignDynSmem = kCapStackSmem * (sizeof(float2) + sizeof(int32_t) + sizeof(float));
+
 constexpr int kDesignThreads = 256;
 
-__global__ void __launch_bounds__(kDesignThreads)
+// One CTA per prompt (and 128 KB of shared memory each): registers are not what limits residency.
+__global__ void __launch_bounds__(kDesignThreads, 1)
     design_kernel(int K, int T_max, const int32_t* __restrict__ L, const float* __restrict__ gamma,
                   const float* __restrict__ u, double budget, int strategy, double param, uint64_t* __restrict__ q,
                   double* __restrict__ xi_out, DesignWs ws, uint32_t* status) {
@@ -289,9 +389,12 @@ __global__ void __launch_bounds__(kDesignThreads)
   __shared__ long long red_l[kDesignThreads / 32];
   __shared__ int red_i[kDesignThreads / 32];
   __shared__ double lam_s;
-  __shared__ int found_s;
+  __shared__ int found_s, found_lane_s, ncand_s, nnear_s, tdef_s;
+  __shared__ volatile int s0_ok_s, s0_skip_s;
+  __shared__ int cand_s[kMaxNearCap + 1];
   __shared__ int nb_s[kCapLanes];
   __shared__ double den_s[kCapLanes];
+  extern __shared__ double dyn_smem[];    // the status pass's stack (kDesignDynSmem bytes)
   const int lane = tid & 31, wid = tid >> 5;
   double* w = ws.w + static_cast<int64_t>(p) * T_max;
   double* xi = ws.xi + static_cast<int64_t>(p) * T_max;
@@ -343,21 +446,109 @@ __global__ void __launch_bounds__(kDesignThreads)
     for (int t = tid; t < Tp; t += kDesignThreads) w[t] = wm > 0.0 ? (w[t] > fl ? w[t] : fl) : 1.0;
     __syncthreads();
     if (strategy == PS_DESIGN_OPTIMIZED) {
-      // The smallest saturated prefix s whose suffix design (budget B - s) starts at or below 1.
-      // The first round tries s = 0 alone; later rounds try 32 consecutive prefixes, one per lane
-      // of warp 0, each with its own stack. All threads then take the blocks' scores
-      // s_m = sqrt(W_m / n_m); each lane sums den = sum_m n_m s_m in block order, and the first
-      // lane (smallest s) whose design starts at or below 1 settles the search.
+      // The smallest saturated prefix s whose suffix design (budget B - s) starts at or below 1,
+      // decided by the definition's exact rounded sequence: for a candidate s, a lane of warp 0 pools
+      // w[s..T) into its own stack; all threads take the blocks' scores s_m = sqrt(W_m / n_m); the
+      // lane sums den = sum_m n_m s_m in block order and tests (B - s) s_1 / den <= 1. Candidates:
+      // the prefixes the status pass puts within the band of 1, then the first clearly below it, in
+      // increasing order; the first that passes is the answer. (If the band holds too many, or none
+      // passes, the search falls back to trying every prefix in order, 32 at a time.)
       const int64_t sbase = static_cast<int64_t>(p) * T_max * kCapLanes;
       double* bW = ws.bW + sbase;
       double* bs = ws.bs + sbase;
       int32_t* bn = ws.bn + sbase;
-      if (tid == 0) found_s = -1;
-      int base = 0;
-      for (int width = 1; base < Tp; base += width, width = kCapLanes) {
+      // xi is written last; meanwhile its 8 Tp bytes hold the scaled weights of the status pass
+      // (floats, [0, Tp)) and the statuses (floats, [Tp, 2 Tp))
+      float* wsc = reinterpret_cast<float*>(xi);
+      float* status = wsc + Tp;
+      {
+        const double inv = 1.0 / (wm > 0.0 ? wm : 1.0);
+        for (int t = tid; t < Tp; t += kDesignThreads) wsc[t] = static_cast<float>(w[t] * inv);
+      }
+      // s = 0 first, exactly (small budgets end here), on warp 0; meanwhile warp 1 runs the status
+      // pass for every other prefix on a stack of its own (shared memory, then lane 31's slots), and
+      // stops as soon as s = 0 has qualified.
+      if (tid == 0) {
+        found_s = -1;
+        nnear_s = 0;
+        ncand_s = 0;
+        s0_ok_s = 0;
+        s0_skip_s = 0;
+      }
+      __syncthreads();
+      if (wid == 0) {
+        // (abandoned when the status pass, finished first, puts s = 0 clearly above the cap)
+        if (lane == 0) nb_s[0] = pav_stack_dev(w, Tp, bW, bn, &s0_skip_s);
+        __syncwarp();
+        const int nb0 = nb_s[0];
+        for (int m = lane; m < nb0; m += 32)
+          bs[m * kCapLanes] = __dsqrt_rn(__ddiv_rn(bW[m * kCapLanes], static_cast<double>(bn[m * kCapLanes])));
+        __syncwarp();
+        if (lane == 0) {
+          double den = 0.0;
+          for (int m = 0; m < nb0; ++m)
+            den = __dadd_rn(den, __dmul_rn(static_cast<double>(bn[m * kCapLanes]), bs[m * kCapLanes]));
+          den_s[0] = den;
+          if (nb0 > 0 && __ddiv_rn(__dmul_rn(Bp, bs[0]), den) <= 1.0) {
+            found_s = 0;
+            found_lane_s = 0;
+            s0_ok_s = 1;
+          }
+        }
+      }
+      if (wid == 1 && lane == 0) {
+        float2* sW = reinterpret_cast<float2*>(dyn_smem);
+        int32_t* sn = reinterpret_cast<int32_t*>(sW + kCapStackSmem);
+        float* sr = reinterpret_cast<float*>(sn + kCapStackSmem);
+        cap_status_pass(wsc, Tp, Bp, sW, sn, sr, bW + (kCapLanes - 1), bn + (kCapLanes - 1),
+                        bs + (kCapLanes - 1), status, &s0_ok_s);
+        if (!s0_ok_s && status[0] == 0.f) s0_skip_s = 1;
+      }
+      __syncthreads();
+      int td = Tp;
+      for (int t = 1 + tid; t < Tp; t += kDesignThreads)
+        if (status[t] == 2.f) {
+          td = t;
+          break;
+        }
+#pragma unroll
+      for (int o = 16; o >= 1; o >>= 1) td = min(td, __shfl_xor_sync(0xffffffffu, td, o));
+      if (lane == 0) red_i[wid] = td;
+      __syncthreads();
+      if (tid == 0) {
+        int m = Tp;
+        for (int i = 0; i < kDesignThreads / 32; ++i) m = min(m, red_i[i]);
+        tdef_s = m;
+      }
+      __syncthreads();
+      const int tdef = tdef_s;
+      if (found_s < 0)
+        for (int t = 1 + tid; t < tdef; t += kDesignThreads)
+          if (status[t] == 1.f) {
+            const int i = atomicAdd(&nnear_s, 1);
+            if (i < kMaxNearCap) cand_s[i] = t;
+          }
+      __syncthreads();
+      if (tid == 0 && found_s < 0) {
+        const int n = min(nnear_s, kMaxNearCap);
+        for (int i = 1; i < n; ++i) {          // the few near-band prefixes, in increasing order
+          const int v = cand_s[i];
+          int j = i - 1;
+          while (j >= 0 && cand_s[j] > v) {
+            cand_s[j + 1] = cand_s[j];
+            --j;
+          }
+          cand_s[j + 1] = v;
+        }
+        ncand_s = nnear_s > kMaxNearCap ? 0 : n + (tdef < Tp ? 1 : 0);
+        if (tdef < Tp && nnear_s <= kMaxNearCap) cand_s[n] = tdef;
+      }
+      __syncthreads();
+      // One round: lanes l < width try the prefixes start(l); sets found_s / found_lane_s.
+      auto try_prefixes = [&](int width, auto start) {
         if (wid == 0) {
-          const int st = base + lane;
-          nb_s[lane] = (lane < width && st < Tp) ? pav_stack_dev(w + st, Tp - st, bW + lane, bn + lane) : 0;
+          const int st = lane < width ? start(lane) : Tp;
+          nb_s[lane] = st < Tp ? pav_stack_dev(w + st, Tp - st, bW + lane, bn + lane) : 0;
         }
         __syncthreads();
         for (int l = 0; l < width; ++l)
@@ -366,9 +557,9 @@ __global__ void __launch_bounds__(kDesignThreads)
                 __dsqrt_rn(__ddiv_rn(bW[m * kCapLanes + l], static_cast<double>(bn[m * kCapLanes + l])));
         __syncthreads();
         if (wid == 0) {
-          const int st = base + lane;
+          const int st = lane < width ? start(lane) : Tp;
           bool ok = false;
-          if (lane < width && st < Tp) {
+          if (st < Tp) {
             double den = 0.0;
             for (int m = 0; m < nb_s[lane]; ++m)
               den = __dadd_rn(den, __dmul_rn(static_cast<double>(bn[m * kCapLanes + lane]), bs[m * kCapLanes + lane]));
@@ -376,17 +567,26 @@ __global__ void __launch_bounds__(kDesignThreads)
             ok = __ddiv_rn(__dmul_rn(__dsub_rn(Bp, static_cast<double>(st)), bs[lane]), den) <= 1.0;
           }
           const unsigned m = __ballot_sync(0xffffffffu, ok);
-          if (lane == 0 && m != 0u) found_s = base + __ffs(m) - 1;
+          if (lane == 0 && m != 0u) {
+            found_lane_s = __ffs(m) - 1;
+            found_s = start(found_lane_s);
+          }
         }
         __syncthreads();
-        if (found_s >= 0) break;
-      }
+      };
+      const int ncand = ncand_s;
+      for (int c0 = 0; c0 < ncand && found_s < 0; c0 += kCapLanes)
+        try_prefixes(min(kCapLanes, ncand - c0), [&](int l) { return cand_s[c0 + l]; });
+      // the exact scan over every prefix: only when the band held too many prefixes or no candidate
+      // passed, which the status pass's accuracy rules out in practice
+      for (int base = 1; found_s < 0 && base < Tp; base += kCapLanes)
+        try_prefixes(kCapLanes, [&](int l) { return base + l; });
       const int found = found_s;
       if (found < 0) {
         for (int t = tid; t < Tp; t += kDesignThreads) xi[t] = 1.0;
       } else {
-        // the design of lane l = found - base: block starts by a scan, then every block in parallel
-        const int l = found - base;
+        // the design of the lane that found it: block starts by a scan, then every block in parallel
+        const int l = found_lane_s;
         const int nb = nb_s[l];
         const double Bs = __dsub_rn(Bp, static_cast<double>(found));
         const double den = den_s[l];
@@ -691,7 +891,10 @@ int ps_design_cutoffs(int P, int K, int T_max, const int32_t* L, const float* ga
     return PS_ERR_WORKSPACE;
   cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
   if (cudaMemsetAsync(ws, 0, kWsHeader, s) != cudaSuccess) return PS_ERR_CUDA;
-  design_kernel<<<P, kDesignThreads, 0, s>>>(K, T_max, L, gamma_full, u, budget, strategy, param, q, xi,
+  if (cudaFuncSetAttribute(design_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                           static_cast<int>(kDesignDynSmem)) != cudaSuccess)
+    return PS_ERR_CUDA;
+  design_kernel<<<P, kDesignThreads, kDesignDynSmem, s>>>(K, T_max, L, gamma_full, u, budget, strategy, param, q, xi,
                                               design_ws(ws, P, K, T_max), static_cast<uint32_t*>(ws));
   return cudaGetLastError() == cudaSuccess ? PS_OK : PS_ERR_CUDA;
 }

@@ -47,6 +47,64 @@ def test_design_masses_bit_exact(name, budget, strategy):
         assert np.array_equal(q, q_ref)
 
 
+@pytest.mark.parametrize("name,budget", [("7b", 2048.0), ("long", 8192.0), ("mid", 150.0), ("tiny_bf16", 200.0)])
+def test_capped_design_at_budgets_that_saturate_long_prefixes(name, budget):
+    # budgets whose designs saturate hundreds to thousands of leading steps at xi = 1 (the cap of
+    # Appendix F): the kernel locates the prefix from one pass of pooling from the right and decides
+    # the candidates near the cap exactly; the masses must still equal the oracle's linear scan
+    cfg = get_config(name)
+    L = draw_lengths(cfg)
+    gamma, u = draw_design_inputs(cfg, L)
+    q, xi = _gpu_design(cfg, L, gamma, u, budget, "optimized")
+    q_ref, xi_ref = design.design_cutoff_masses(L, cfg.K, gamma, u, budget, "optimized")
+    assert np.array_equal(xi, xi_ref), np.abs(xi - xi_ref).max()
+    assert np.array_equal(q, q_ref)
+    assert (xi == 1.0).sum() > 0
+
+
+def _crafted_design(vectors, budget):
+    """One prompt per weight vector, each a group of one completion (K = 1), so gamma_bar, and with
+    no u the weights, are the vector itself (floored at 1e-12 of the maximum)."""
+    from types import SimpleNamespace
+    L = np.array([len(v) for v in vectors], dtype=np.int32)
+    gamma = np.concatenate([np.asarray(v, dtype=np.float32) for v in vectors])
+    q, xi = _gpu_design(SimpleNamespace(P=len(vectors), K=1), L, gamma, None, budget, "optimized")
+    q_ref, xi_ref = design.design_cutoff_masses(L, 1, gamma, None, budget, "optimized")
+    assert np.array_equal(xi, xi_ref), np.abs(xi - xi_ref).max()
+    assert np.array_equal(q, q_ref)
+    return xi
+
+
+def test_capped_design_crafted_cases():
+    # (0, 100, 1 x 10) with B = 3.2: saturating nothing already meets the cap (the pooled block
+    # {0, 1} starts at 0.94), while saturating one step does not (1.1): qualifying prefixes are not
+    # monotone in their length, so the search must not bisect
+    xi = _crafted_design([[0.0, 100.0] + [1.0] * 10], 3.2)
+    assert xi[0, 0] < 1.0
+    # uniform weights: every suffix design starts at exactly B' / T', i.e. at 1 when B = T (the
+    # decision sits on the cap); and below it
+    for B in (12.0, 11.5, 3.0):
+        _crafted_design([[1.0] * 12, [2.0] * 7, [5.0] * 12], B)
+    # steep fronts: geometric weights, a plateau, a ramp up, pooled violators after the cap
+    rng = np.random.default_rng(7)
+    vecs = [[2.0 ** -t for t in range(60)], [50.0] * 5 + [1.0] * 40, list(np.linspace(1, 30, 50)),
+            list(np.sort(rng.uniform(0.1, 9.0, 80))[::-1] ** 3 * rng.uniform(0.5, 1.5, 80))]
+    for B in (2.0, 10.0, 25.0, 44.0, 59.0, 60.0):
+        _crafted_design(vecs, B)
+
+
+@pytest.mark.parametrize("seed", range(4))
+def test_capped_design_random_steep_weights(seed):
+    rng = np.random.default_rng(50 + seed)
+    vecs = []
+    for _ in range(24):
+        T = int(rng.integers(2, 400))
+        w = np.sort(rng.lognormal(0.0, 2.0, T))[::-1] * rng.lognormal(0.0, 0.5, T)
+        vecs.append(w)
+    for B in (1.5, 17.0, 130.0, 399.0):
+        _crafted_design(vecs, B)
+
+
 @pytest.mark.parametrize("name,budget", [("mid", 40.0), ("7b", 128.0)])
 def test_time_prior_design(name, budget):
     cfg = get_config(name)
