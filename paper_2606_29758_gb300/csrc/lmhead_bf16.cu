@@ -16,6 +16,21 @@
 namespace psk {
 
 // ============================================================================= epilogues
+// Value j of a 32-column slice of accumulator registers, picked by a select tree on the bits of j
+// (a dynamic index into the registers would move them to local memory).
+static __device__ __forceinline__ float pick32(const uint32_t (&r)[32], int j) {
+  float a[16];
+#pragma unroll
+  for (int i = 0; i < 16; ++i) a[i] = __uint_as_float((j & 1) ? r[2 * i + 1] : r[2 * i]);
+#pragma unroll
+  for (int i = 0; i < 8; ++i) a[i] = (j & 2) ? a[2 * i + 1] : a[2 * i];
+#pragma unroll
+  for (int i = 0; i < 4; ++i) a[i] = (j & 4) ? a[2 * i + 1] : a[2 * i];
+#pragma unroll
+  for (int i = 0; i < 2; ++i) a[i] = (j & 8) ? a[2 * i + 1] : a[2 * i];
+  return (j & 16) ? a[1] : a[0];
+}
+
 struct FwdLseEpi {
   struct Params {
     const int32_t* tok;
@@ -36,9 +51,14 @@ struct FwdLseEpi {
                                                const uint32_t (&r)[32]) {
     if (col0 >= p.N) return;
     float x[32];
-    const int nv = p.N - col0;
+    if (col0 + 32 <= p.N) {
 #pragma unroll
-    for (int j = 0; j < 32; ++j) x[j] = (j < nv) ? __uint_as_float(r[j]) * kLog2e : -INFINITY;
+      for (int j = 0; j < 32; ++j) x[j] = __uint_as_float(r[j]) * kLog2e;
+    } else {   // the vocabulary's ragged last slice
+      const int nv = p.N - col0;
+#pragma unroll
+      for (int j = 0; j < 32; ++j) x[j] = (j < nv) ? __uint_as_float(r[j]) * kLog2e : -INFINITY;
+    }
     float c0 = fmaxf(x[0], x[1]), c1 = fmaxf(x[2], x[3]);
 #pragma unroll
     for (int j = 4; j < 32; j += 4) {
@@ -46,23 +66,17 @@ struct FwdLseEpi {
       c1 = fmaxf(c1, fmaxf(x[j + 2], x[j + 3]));
     }
     const int rel = st.tok - col0;
-    if (static_cast<unsigned>(rel) < 32u) {
-      float zt = 0.f;
-#pragma unroll
-      for (int j = 0; j < 32; ++j)
-        if (j == rel) zt = __uint_as_float(r[j]);
-      p.ztok[row] = zt;
-    }
+    if (static_cast<unsigned>(rel) < 32u) p.ztok[row] = pick32(r, rel);
     const float mn = fmaxf(st.m2, fmaxf(c0, c1));
     float a0 = 0.f, a1 = 0.f, a2 = 0.f, a3 = 0.f;
 #pragma unroll
     for (int j = 0; j < 32; j += 4) {
-      a0 += exp2f(x[j] - mn);
-      a1 += exp2f(x[j + 1] - mn);
-      a2 += exp2f(x[j + 2] - mn);
-      a3 += exp2f(x[j + 3] - mn);
+      a0 += ex2_ftz(x[j] - mn);
+      a1 += ex2_ftz(x[j + 1] - mn);
+      a2 += ex2_ftz(x[j + 2] - mn);
+      a3 += ex2_ftz(x[j + 3] - mn);
     }
-    st.s = st.s * exp2f(st.m2 - mn) + ((a0 + a1) + (a2 + a3));
+    st.s = st.s * ex2_ftz(st.m2 - mn) + ((a0 + a1) + (a2 + a3));
     st.m2 = mn;
   }
   static __device__ __forceinline__ void end_unit(const Params& p, State& st, int row, int split) {
@@ -96,9 +110,14 @@ struct FwdProxyEpi {
                                                const uint32_t (&r)[32]) {
     if (col0 >= p.N) return;
     float x[32];
-    const int nv = p.N - col0;
+    if (col0 + 32 <= p.N) {
 #pragma unroll
-    for (int j = 0; j < 32; ++j) x[j] = (j < nv) ? __uint_as_float(r[j]) * kLog2e : -INFINITY;
+      for (int j = 0; j < 32; ++j) x[j] = __uint_as_float(r[j]) * kLog2e;
+    } else {   // the vocabulary's ragged last slice
+      const int nv = p.N - col0;
+#pragma unroll
+      for (int j = 0; j < 32; ++j) x[j] = (j < nv) ? __uint_as_float(r[j]) * kLog2e : -INFINITY;
+    }
     float c0 = fmaxf(x[0], x[1]), c1 = fmaxf(x[2], x[3]);
 #pragma unroll
     for (int j = 4; j < 32; j += 4) {
@@ -120,13 +139,13 @@ struct FwdProxyEpi {
     float a0 = 0.f, a1 = 0.f, b0 = 0.f, b1 = 0.f;
 #pragma unroll
     for (int j = 0; j < 32; j += 2) {
-      const float e0 = exp2f(x[j] - mn), e1 = exp2f(x[j + 1] - mn);
+      const float e0 = ex2_ftz(x[j] - mn), e1 = ex2_ftz(x[j + 1] - mn);
       a0 += e0;
       a1 += e1;
       b0 = fmaf(e0, e0, b0);
       b1 = fmaf(e1, e1, b1);
     }
-    const float f = exp2f(st.m2 - mn);
+    const float f = ex2_ftz(st.m2 - mn);
     st.s1 = st.s1 * f + (a0 + a1);
     st.s2 = st.s2 * (f * f) + (b0 + b1);
     st.m2 = mn;
@@ -161,19 +180,6 @@ struct FwdProxyTopkEpi {
       st.v[j] = -INFINITY;
       st.id[j] = -1;
     }
-  }
-  // Value j of the slice, picked by a select tree on the bits of j (keeps r in registers).
-  static __device__ __forceinline__ float pick32(const uint32_t (&r)[32], int j) {
-    float a[16];
-#pragma unroll
-    for (int i = 0; i < 16; ++i) a[i] = __uint_as_float((j & 1) ? r[2 * i + 1] : r[2 * i]);
-#pragma unroll
-    for (int i = 0; i < 8; ++i) a[i] = (j & 2) ? a[2 * i + 1] : a[2 * i];
-#pragma unroll
-    for (int i = 0; i < 4; ++i) a[i] = (j & 4) ? a[2 * i + 1] : a[2 * i];
-#pragma unroll
-    for (int i = 0; i < 2; ++i) a[i] = (j & 8) ? a[2 * i + 1] : a[2 * i];
-    return (j & 16) ? a[1] : a[0];
   }
   static __device__ __forceinline__ void chunk(const Params& p, State& st, int row, int col0,
                                                const uint32_t (&r)[32]) {
@@ -250,14 +256,24 @@ struct BwdDzEpi {
 #pragma unroll
       for (int j = 0; j < 16; ++j) pk[j] = 0u;
     } else {
+      // dZ_v = coef (1[v = o] - p_v). The chosen column o lies in one slice of the ~600 a row has:
+      // every other slice is -coef p_v, without the test per column.
+      const float nc = -st.coef;
       const int rel = st.tok - col0;
+      if (static_cast<unsigned>(rel) < 32u) {
 #pragma unroll
-      for (int j = 0; j < 16; ++j) {
-        const float p0 = exp2f(fmaf(__uint_as_float(r[2 * j]), kLog2e, -st.lse2));
-        const float p1 = exp2f(fmaf(__uint_as_float(r[2 * j + 1]), kLog2e, -st.lse2));
-        const float d0 = fmaf(-st.coef, p0, rel == 2 * j ? st.coef : 0.f);
-        const float d1 = fmaf(-st.coef, p1, rel == 2 * j + 1 ? st.coef : 0.f);
-        pk[j] = pack_bf16x2(d0, d1);
+        for (int j = 0; j < 16; ++j) {
+          const float p0 = ex2_ftz(fmaf(__uint_as_float(r[2 * j]), kLog2e, -st.lse2));
+          const float p1 = ex2_ftz(fmaf(__uint_as_float(r[2 * j + 1]), kLog2e, -st.lse2));
+          pk[j] = pack_bf16x2(fmaf(nc, p0, rel == 2 * j ? st.coef : 0.f), fmaf(nc, p1, rel == 2 * j + 1 ? st.coef : 0.f));
+        }
+      } else {
+#pragma unroll
+        for (int j = 0; j < 16; ++j) {
+          const float p0 = ex2_ftz(fmaf(__uint_as_float(r[2 * j]), kLog2e, -st.lse2));
+          const float p1 = ex2_ftz(fmaf(__uint_as_float(r[2 * j + 1]), kLog2e, -st.lse2));
+          pk[j] = pack_bf16x2(nc * p0, nc * p1);
+        }
       }
     }
     __nv_bfloat16* dst = p.dz + static_cast<int64_t>(row) * p.ldz + col0;
