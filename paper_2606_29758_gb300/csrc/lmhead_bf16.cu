@@ -32,6 +32,7 @@ static __device__ __forceinline__ float pick32(const uint32_t (&r)[32], int j) {
 }
 
 struct FwdLseEpi {
+  static constexpr bool kTmaStore = false;
   struct Params {
     const int32_t* tok;
     int M, N;
@@ -90,6 +91,7 @@ struct FwdLseEpi {
 // that ||e_o - p||^2 = (r1^2 + r2) / (e_o + r1)^2 keeps its relative accuracy when p(o) -> 1
 // (1 - 2 p(o) + ||p||^2 would cancel there).
 struct FwdProxyEpi {
+  static constexpr bool kTmaStore = false;
   struct Params {
     const int32_t* tok;
     int M, N;
@@ -160,6 +162,7 @@ struct FwdProxyEpi {
 // registers; only the values of a 32-column slice above the current 16th value are inserted.
 constexpr int kTopK = 16;
 struct FwdProxyTopkEpi {
+  static constexpr bool kTmaStore = false;
   struct Params {
     const int32_t* tok;
     int M, N;
@@ -224,19 +227,23 @@ struct FwdProxyTopkEpi {
   }
 };
 
+// Recomputed logits -> dZ = coef (onehot - softmax) in bf16, stored through TMA: each epilogue warp
+// writes its 32 rows x 32 columns of a slice into a staging buffer and one lane issues the tensor
+// store (coalesced 64-byte row segments; rows beyond the chunk and columns beyond V are clipped by
+// the store itself).
 struct BwdDzEpi {
+  static constexpr bool kTmaStore = true;
   struct Params {
     const int32_t* tok;
     const float* lse;
     const float* coef;
     int M, N;
-    __nv_bfloat16* dz;
-    int64_t ldz;
   };
   struct State {
     float lse2, coef;
     int tok;
   };
+  static __device__ __forceinline__ int cols(const Params& p) { return p.N; }
   static __device__ __forceinline__ void begin_unit(const Params& p, State& st, int row, int) {
     if (row < p.M) {
       st.tok = __ldg(p.tok + row);
@@ -245,12 +252,13 @@ struct BwdDzEpi {
     } else {
       st.tok = -1;
       st.lse2 = 0.f;
-      st.coef = 0.f;
+      st.coef = 0.f;   // rows past the chunk: zeros, which the store clips anyway
     }
   }
-  static __device__ __forceinline__ void chunk(const Params& p, State& st, int row, int col0,
-                                               const uint32_t (&r)[32]) {
-    if (row >= p.M || col0 >= p.N) return;
+  // This lane's row of the slice: 32 bf16 = four 16-byte units, unit u at position u ^ ((lane >> 1) & 3)
+  // of the lane's 64-byte row in `buf` (the 64-byte swizzle of the dZ tensor map).
+  static __device__ __forceinline__ void chunk_to_smem(const Params& p, State& st, int, int col0,
+                                                       const uint32_t (&r)[32], uint8_t* buf, int lane) {
     uint32_t pk[16];
     if (st.coef == 0.f) {
 #pragma unroll
@@ -276,23 +284,16 @@ struct BwdDzEpi {
         }
       }
     }
-    __nv_bfloat16* dst = p.dz + static_cast<int64_t>(row) * p.ldz + col0;
-    if (col0 + 32 <= p.N) {
-      uint4* d4 = reinterpret_cast<uint4*>(dst);
+    uint4* dst = reinterpret_cast<uint4*>(buf + lane * 64);
+    const int x = (lane >> 1) & 3;
 #pragma unroll
-      for (int q = 0; q < 4; ++q) d4[q] = make_uint4(pk[4 * q], pk[4 * q + 1], pk[4 * q + 2], pk[4 * q + 3]);
-    } else {
-      const int nv = p.N - col0;
-      unsigned short* d16 = reinterpret_cast<unsigned short*>(dst);
-#pragma unroll
-      for (int j = 0; j < 32; ++j)
-        if (j < nv) d16[j] = static_cast<unsigned short>((j & 1) ? (pk[j >> 1] >> 16) : (pk[j >> 1] & 0xFFFFu));
-    }
+    for (int q = 0; q < 4; ++q) dst[q ^ x] = make_uint4(pk[4 * q], pk[4 * q + 1], pk[4 * q + 2], pk[4 * q + 3]);
   }
   static __device__ __forceinline__ void end_unit(const Params&, State&, int, int) {}
 };
 
 struct StoreF32Epi {
+  static constexpr bool kTmaStore = false;
   struct Params {
     float* out;
     int64_t ld;
@@ -350,7 +351,8 @@ static EncodeTiledFn encode_fn() {
 
 // 2-D bf16 tensor [outer][inner] with row pitch `pitch_bytes`, 128-byte swizzled boxes.
 static bool make_map(CUtensorMap* m, const void* base, uint64_t inner, uint64_t outer, uint64_t pitch_bytes,
-                     uint32_t box_inner, uint32_t box_outer) {
+                     uint32_t box_inner, uint32_t box_outer,
+                     CUtensorMapSwizzle swizzle = CU_TENSOR_MAP_SWIZZLE_128B) {
   EncodeTiledFn enc = encode_fn();
   if (!enc) return false;
   if ((reinterpret_cast<uintptr_t>(base) & 15) || (pitch_bytes & 15)) return false;
@@ -359,7 +361,7 @@ static bool make_map(CUtensorMap* m, const void* base, uint64_t inner, uint64_t 
   const cuuint32_t box[2] = {box_inner, box_outer};
   const cuuint32_t estr[2] = {1, 1};
   return enc(m, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<void*>(base), dims, strides, box, estr,
-             CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+             CU_TENSOR_MAP_INTERLEAVE_NONE, swizzle, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
              CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
 }
 
@@ -373,9 +375,9 @@ static bool map_mnmajor(CUtensorMap* m, const void* base, int64_t K, int64_t MN,
 }
 
 template <bool A_MN, bool B_MN, class Epi, int HALVES = 1>
-static int launch_gemm_single(const CUtensorMap& ta, const CUtensorMap& tb, int64_t M, int64_t N, int64_t K,
-                              int splits, int band_m, const typename Epi::Params& ep, uint32_t* status,
-                              cudaStream_t s) {
+static int launch_gemm_single(const CUtensorMap& ta, const CUtensorMap& tb, const CUtensorMap& tc, int64_t M,
+                              int64_t N, int64_t K, int splits, int band_m, const typename Epi::Params& ep,
+                              uint32_t* status, cudaStream_t s) {
   Sched sc;
   sc.m_blocks = static_cast<int>((M + kBM * HALVES - 1) / (kBM * HALVES));
   sc.n_blocks = static_cast<int>((N + kBN - 1) / kBN);
@@ -391,7 +393,7 @@ static int launch_gemm_single(const CUtensorMap& ta, const CUtensorMap& tb, int6
       cudaSuccess)
     return PS_ERR_CUDA;
   const int grid = sc.num_units < num_sms_current() ? sc.num_units : num_sms_current();
-  kern<<<grid, kGemmThreads, smem, s>>>(ta, tb, sc, ep, status, kDefaultTimeoutNs);
+  kern<<<grid, kGemmThreads, smem, s>>>(ta, tb, tc, sc, ep, status, kDefaultTimeoutNs);
   return cudaGetLastError() == cudaSuccess ? PS_OK : PS_ERR_CUDA;
 }
 
@@ -444,7 +446,7 @@ template <bool A_MN, bool B_MN, class Epi>
 static int launch_gemm(bool pair, const CUtensorMap& ta, const CUtensorMap& tb, int64_t M, int64_t N, int64_t K,
                        int splits, int band_m, const typename Epi::Params& ep, uint32_t* status, cudaStream_t s) {
   return pair ? launch_gemm_pair<A_MN, B_MN, Epi>(ta, tb, M, N, K, splits, band_m, ep, status, s)
-              : launch_gemm_single<A_MN, B_MN, Epi>(ta, tb, M, N, K, splits, band_m, ep, status, s);
+              : launch_gemm_single<A_MN, B_MN, Epi>(ta, tb, ta, M, N, K, splits, band_m, ep, status, s);
 }
 
 int fwd_tile_splits_bf16(int V) { return (V + kBN - 1) / kBN; }
@@ -471,11 +473,11 @@ static int choose_splits(int64_t m_blocks, int64_t n_blocks, int workers, int mi
 // 256-row B tile. (The CTA-pair kernel, reached only through the GEMM test hook, has each CTA
 // load half of it, 128 rows; see gemm_bf16.)
 constexpr uint32_t kBRowsBox = kBN;
-// Tile height of the forward and of the logit recompute in 128-row halves (see GemmCfg). The
-// forward gains from the wide tile (fewer operand bytes per FLOP) even though its epilogue is
-// then not overlapped; the recompute, whose epilogue also writes dZ, does better with
-// 128-row tiles and double-buffered accumulators (7B-shaped step, measured back to back).
-constexpr int kRecHalves = 1;
+// Tile height of the logit recompute in 128-row halves (see GemmCfg). The wide tile moves a third
+// fewer operand bytes per FLOP (about 0.8 vs 0.95 pJ per FLOP at the power cap) but does not overlap
+// its epilogue with the next tile; with dZ stored through TMA it is the faster of the two (7B-shaped
+// backward 381.4 vs 382.8 ms, and 387.7 ms with per-thread stores of 128-row tiles, back to back).
+constexpr int kRecHalves = 2;
 // The forward's (and score proxy's) tile height depends on the hidden size: its K loop is d long,
 // while the epilogue of a wide tile is a fixed cost that is not overlapped. Measured back to back:
 // at d = 3584 the wide tile is 1% faster, at d = 1536 the 128-row tile is 7% faster.
@@ -516,8 +518,8 @@ int fwd_gemm_bf16(int64_t N, int d, int V, const void* Hpk, const void* W, const
   const int workers = num_sms_current();
   const int band = splits == fwd_tile_splits_bf16(V) ? fwd_band_max(d) : (workers + splits - 1) / splits;
   if (halves == 1)
-    return launch_gemm_single<false, false, FwdLseEpi, 1>(ta, tb, N, V, d, splits, band, ep, status, s);
-  return launch_gemm_single<false, false, FwdLseEpi, 2>(ta, tb, N, V, d, splits, band, ep, status, s);
+    return launch_gemm_single<false, false, FwdLseEpi, 1>(ta, tb, ta, N, V, d, splits, band, ep, status, s);
+  return launch_gemm_single<false, false, FwdLseEpi, 2>(ta, tb, ta, N, V, d, splits, band, ep, status, s);
 }
 
 // Bands (row blocks walked together) of the backward GEMMs. Recompute: 48 row blocks share
@@ -538,8 +540,8 @@ int proxy_gemm_bf16(int64_t N, int d, int V, const void* Hrows, const void* W, c
   const int workers = num_sms_current();
   const int band = splits == fwd_tile_splits_bf16(V) ? fwd_band_max(d) : (workers + splits - 1) / splits;
   if (halves == 1)
-    return launch_gemm_single<false, false, FwdProxyEpi, 1>(ta, tb, N, V, d, splits, band, ep, status, s);
-  return launch_gemm_single<false, false, FwdProxyEpi, 2>(ta, tb, N, V, d, splits, band, ep, status, s);
+    return launch_gemm_single<false, false, FwdProxyEpi, 1>(ta, tb, ta, N, V, d, splits, band, ep, status, s);
+  return launch_gemm_single<false, false, FwdProxyEpi, 2>(ta, tb, ta, N, V, d, splits, band, ep, status, s);
 }
 
 int proxy_topk_gemm_bf16(int64_t N, int d, int V, const void* Hrows, const void* W, const int32_t* tok,
@@ -552,7 +554,7 @@ int proxy_topk_gemm_bf16(int64_t N, int d, int V, const void* Hrows, const void*
   const int workers = num_sms_current();
   int band = static_cast<int>(kFwdBandL2Bytes / (static_cast<double>(kBM) * d * 2.0));
   if (band < (workers + splits - 1) / splits) band = (workers + splits - 1) / splits;
-  return launch_gemm_single<false, false, FwdProxyTopkEpi, 1>(ta, tb, N, V, d, splits, band, ep, status, s);
+  return launch_gemm_single<false, false, FwdProxyTopkEpi, 1>(ta, tb, ta, N, V, d, splits, band, ep, status, s);
 }
 
 int bwd_chunk_bf16(int64_t rc, int d, int V, const void* Hpk, const void* W, const int32_t* tok,
@@ -563,9 +565,12 @@ int bwd_chunk_bf16(int64_t rc, int d, int V, const void* Hpk, const void* W, con
     CUtensorMap ta, tb;
     if (!map_kmajor(&ta, Hpk, rc, d, d, kBM * kRecHalves) || !map_kmajor(&tb, W, V, d, d, kBRowsBox))
       return PS_ERR_INVALID_ARG;
-    BwdDzEpi::Params ep{tok, lse, coef, static_cast<int>(rc), V, static_cast<__nv_bfloat16*>(dz), ldz};
-    rcode = launch_gemm_single<false, false, BwdDzEpi, kRecHalves>(ta, tb, rc, V, d, 0, kBandRecompute / kRecHalves,
-                                                                    ep, status, s);
+    // dZ [rc][ldz] bf16, written in 32 x 32 boxes from 64-byte-swizzled staging
+    CUtensorMap tz;
+    if (!make_map(&tz, dz, V, rc, ldz * 2, 32, 32, CU_TENSOR_MAP_SWIZZLE_64B)) return PS_ERR_INVALID_ARG;
+    BwdDzEpi::Params ep{tok, lse, coef, static_cast<int>(rc), V};
+    rcode = launch_gemm_single<false, false, BwdDzEpi, kRecHalves>(ta, tb, tz, rc, V, d, 0,
+                                                                    kBandRecompute / kRecHalves, ep, status, s);
     if (rcode != PS_OK) return rcode;
   }
   // dH (K = V) and dW (K = chunk rows) have long K loops: one CTA computes a 256 x 256 tile
@@ -574,14 +579,14 @@ int bwd_chunk_bf16(int64_t rc, int d, int V, const void* Hpk, const void* W, con
     CUtensorMap ta, tb;
     if (!map_kmajor(&ta, dz, rc, V, ldz, 2 * kBM) || !map_mnmajor(&tb, W, V, d, d)) return PS_ERR_INVALID_ARG;
     StoreF32Epi::Params ep{dH, d, static_cast<int>(rc), d, 0};
-    rcode = launch_gemm_single<false, true, StoreF32Epi, 2>(ta, tb, rc, d, V, 0, kBandGrad, ep, status, s);
+    rcode = launch_gemm_single<false, true, StoreF32Epi, 2>(ta, tb, ta, rc, d, V, 0, kBandGrad, ep, status, s);
     if (rcode != PS_OK) return rcode;
   }
   if (dW) {
     CUtensorMap ta, tb;
     if (!map_mnmajor(&ta, dz, rc, V, ldz) || !map_mnmajor(&tb, Hpk, rc, d, d)) return PS_ERR_INVALID_ARG;
     StoreF32Epi::Params ep{dW, d, V, d, dw_accumulate};
-    rcode = launch_gemm_single<true, true, StoreF32Epi, 2>(ta, tb, V, d, rc, 0, kBandGrad, ep, status, s);
+    rcode = launch_gemm_single<true, true, StoreF32Epi, 2>(ta, tb, ta, V, d, rc, 0, kBandGrad, ep, status, s);
     if (rcode != PS_OK) return rcode;
   }
   return PS_OK;
@@ -599,10 +604,10 @@ int gemm_bf16(int M, int N, int K, int a_mn, int b_mn, const void* A, int64_t ld
   StoreF32Epi::Params ep{C, ldc, M, N, accumulate};
   using E = StoreF32Epi;
   if (variant == 2) {
-    if (!a_mn && !b_mn) return launch_gemm_single<false, false, E, 2>(ta, tb, M, N, K, 0, 16, ep, status, s);
-    if (!a_mn && b_mn) return launch_gemm_single<false, true, E, 2>(ta, tb, M, N, K, 0, 16, ep, status, s);
-    if (a_mn && b_mn) return launch_gemm_single<true, true, E, 2>(ta, tb, M, N, K, 0, 16, ep, status, s);
-    return launch_gemm_single<true, false, E, 2>(ta, tb, M, N, K, 0, 16, ep, status, s);
+    if (!a_mn && !b_mn) return launch_gemm_single<false, false, E, 2>(ta, tb, ta, M, N, K, 0, 16, ep, status, s);
+    if (!a_mn && b_mn) return launch_gemm_single<false, true, E, 2>(ta, tb, ta, M, N, K, 0, 16, ep, status, s);
+    if (a_mn && b_mn) return launch_gemm_single<true, true, E, 2>(ta, tb, ta, M, N, K, 0, 16, ep, status, s);
+    return launch_gemm_single<true, false, E, 2>(ta, tb, ta, M, N, K, 0, 16, ep, status, s);
   }
   const bool p = variant == 1;
   if (!a_mn && !b_mn) return launch_gemm<false, false, E>(p, ta, tb, M, N, K, 0, 16, ep, status, s);

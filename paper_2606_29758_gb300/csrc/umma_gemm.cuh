@@ -68,11 +68,17 @@ struct GemmCfg {
   static constexpr int kAccBufs = HALVES == 1 ? 2 : 1;        // accumulator buffers in TMEM
 };
 
+// Epilogues that store through TMA (Epi::kTmaStore) stage each 32-row x 32-column bf16 slice of a
+// warp in shared memory, two buffers per epilogue warp, 64-byte swizzled (a 64-byte row per TMEM
+// lane, its 16-byte units permuted by row bits 1-2, so a warp's stores hit every bank group).
+constexpr int kStageBytes = 32 * 64;
+
 template <int HALVES>
 struct GemmSmemT {
   // 1024-byte aligned tile ring first (128-byte swizzle atoms repeat every 1 KB)
   uint8_t a[GemmCfg<HALVES>::kStagesH][GemmCfg<HALVES>::kABytes];
   uint8_t b[GemmCfg<HALVES>::kStagesH][kTileBBytes];
+  uint8_t stage[4][2][kStageBytes];   // store staging of the four epilogue warps (2 KB-aligned)
   uint64_t full[GemmCfg<HALVES>::kStagesH];
   uint64_t empty[GemmCfg<HALVES>::kStagesH];
   uint64_t tfull[2];
@@ -85,10 +91,12 @@ template <int HALVES>
 constexpr size_t gemm_smem_bytes() { return sizeof(GemmSmemT<HALVES>) + 1024; }  // + alignment slack
 constexpr size_t kGemmSmemBytes = gemm_smem_bytes<1>();
 
+// tmC: the output map of epilogues that store through TMA (unused by the others).
 template <bool A_MN, bool B_MN, class Epi, int HALVES = 1>
 __global__ void __launch_bounds__(kGemmThreads, 1)
     umma_gemm_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmB,
-                     const Sched sched, const typename Epi::Params ep, uint32_t* status, uint64_t timeout_ns) {
+                     const __grid_constant__ CUtensorMap tmC, const Sched sched, const typename Epi::Params ep,
+                     uint32_t* status, uint64_t timeout_ns) {
   using Cfg = GemmCfg<HALVES>;
   constexpr int S = Cfg::kStagesH;
   constexpr int NB = Cfg::kAccBufs;
@@ -220,6 +228,7 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
     const int row_in_tile = quad * 32 + lane;
     typename Epi::State st[HALVES];             // a thread owns row r of each half
     uint32_t tile = 0;
+    uint32_t nstore = 0;                        // TMA-stored slices of this warp
     bool ok = true;
     for (int u = blockIdx.x; ok && u < sched.num_units; u += gridDim.x) {
       int m_blk, split, n0, n1;
@@ -250,7 +259,25 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
               tc_fence_before();
               mbar_arrive(&sm.tempty[acc]);
             }
-            Epi::chunk(ep, st[h], row, nb * kBN + c * 32, r);
+            const int col0 = nb * kBN + c * 32;
+            if constexpr (Epi::kTmaStore) {
+              // the slice goes to a staging buffer, then one lane stores the warp's 32 x 32 box
+              if (col0 < Epi::cols(ep)) {
+                uint8_t* buf = sm.stage[quad][nstore & 1];
+                if (lane == 0) bulk_wait_group_read<1>();   // the store of two slices ago has read it
+                __syncwarp();
+                Epi::chunk_to_smem(ep, st[h], row, col0, r, buf, lane);
+                fence_proxy_async_smem();
+                __syncwarp();
+                if (lane == 0) {
+                  tma_store_2d(&tmC, buf, col0, m_blk * Cfg::kRows + h * kBM + quad * 32);
+                  bulk_commit_group();
+                }
+                ++nstore;
+              }
+            } else {
+              Epi::chunk(ep, st[h], row, col0, r);
+            }
           }
         }
       }
@@ -263,6 +290,8 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
       *abort = 1;
       raise_status(status, PS_DEV_TIMEOUT);
     }
+    // the staged stores must finish reading shared memory (and reach global memory) before exit
+    if (Epi::kTmaStore && lane == 0) bulk_wait_group_all();
   }
 
   tc_fence_before();
