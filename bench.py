@@ -12,9 +12,11 @@ by the max over ranks of the device-timed region). The credited work of a step i
 
     python bench.py [--gpus N] [--steps K] [--warmup W] [--impl ours|reference|torch]
 
-With --gpus N > 1 (launched by torchrun) every rank runs its own replica of the
-workload on its own GPU: the pass has no cross-rank exchange in this form
-(weak scaling). --impl reference times the CPU float64 oracle on bounded samples of
+With --gpus N > 1 (launched by torchrun) the step is data-parallel (weak scaling): every rank
+holds its own batch of the workload's P prompts (global batch N x P), draws the cutoffs of its
+completions by their global index (traj_base = rank x P x K) with the global loss scale
+1/(N P K), and after the backward dW and the loss are summed over the ranks (NCCL all-reduce,
+inside the timed step). --replicas runs N independent replicas without the exchange. --impl reference times the CPU float64 oracle on bounded samples of
 the same workload, on the host cores. --impl torch (context only) runs the head of the same step
 in eager PyTorch with materialised logits.
 """
@@ -124,7 +126,7 @@ def run_ours(args):
     import torch
     import torch.distributed as dist
 
-    from paper_2606_29758_gb300 import InputStager, PassShape, UpdatePass
+    from paper_2606_29758_gb300 import DataParallelUpdate, InputStager, PassShape, UpdatePass
     from synthetic import get_config, make_batch
 
     world, rank, local = _dist()
@@ -137,14 +139,17 @@ def run_ours(args):
     D = b.dev
     tdtype = torch.bfloat16 if cfg.dtype == "bf16" else torch.float32
     shape = PassShape(cfg.P, cfg.K, b.T_max, cfg.d, cfg.V, b.total_len, tdtype, args.chunk_rows)
-    up = UpdatePass(shape, device=dev, eps=cfg.eps, loss_scale=cfg.loss_scale)
+    # data-parallel: every rank's completions are a slice of one global batch of world x P prompts
+    dp = world > 1 and not args.replicas
+    up = UpdatePass(shape, device=dev, eps=cfg.eps, loss_scale=cfg.loss_scale / world if dp else cfg.loss_scale)
+    dpu = DataParallelUpdate(up, traj_base=rank * cfg.B if dp else 0)
     stream = torch.cuda.current_stream()
     seed = cfg.seed
 
     def step(i, ev=None):
         if ev is not None:
             ev[0].record(stream)
-        up.sample(D["q"], D["L"], seed, i)
+        up.sample(D["q"], D["L"], seed, i, traj_base=dpu.traj_base)
         if ev is not None:
             ev[1].record(stream)
         n = up.pack(D["L"], D["R"], D["tok_full"], D["oldlogp_full"], D["hid_full"])
@@ -156,6 +161,10 @@ def run_ours(args):
         up.backward(D["W"])
         if ev is not None:
             ev[4].record(stream)
+        if dp:
+            dpu.exchange()
+        if ev is not None:
+            ev[5].record(stream)
         return n
 
     def barrier():
@@ -173,7 +182,7 @@ def run_ours(args):
         clocks = ClockSampler(local)
         clocks.start()
         time.sleep(0.3)
-        evs = [[torch.cuda.Event(enable_timing=True) for _ in range(5)] for _ in range(args.steps)]
+        evs = [[torch.cuda.Event(enable_timing=True) for _ in range(6)] for _ in range(args.steps)]
         barrier()
         t0 = torch.cuda.Event(enable_timing=True)
         t1 = torch.cuda.Event(enable_timing=True)
@@ -185,7 +194,7 @@ def run_ours(args):
         barrier()
         clk = clocks.stop()
         up.check_status()
-        per = np.array([[e[j].elapsed_time(e[j + 1]) for j in range(4)] for e in evs])   # sample, pack, fwd, bwd
+        per = np.array([[e[j].elapsed_time(e[j + 1]) for j in range(5)] for e in evs])   # sample, pack, fwd, bwd, exchange
         return t0.elapsed_time(t1), step_rows, per, clk
 
     ms, step_rows, per, clk = timed_region(0)
@@ -241,10 +250,12 @@ def run_ours(args):
         for i in range(n_steps):
             X = stager.acquire(j, stream)
             nxt = stager.stage(host) if i + 1 < n_steps else None
-            up.sample(X["q"], X["L"], seed, base + i)
+            up.sample(X["q"], X["L"], seed, base + i, traj_base=dpu.traj_base)
             total += up.pack(X["L"], X["R"], X["tok_full"], X["oldlogp_full"], X["hid_full"])
             up.forward(D["W"])
             up.backward(D["W"])
+            if dp:
+                dpu.exchange()
             stager.release(j, stream)
             loss_h[i].copy_(up.loss[0], non_blocking=True)
             stream.synchronize()
@@ -368,7 +379,9 @@ def run_ours(args):
                    "bwd_chunk_rows": args.chunk_rows,
                    "l2": f"inputs larger than L2 (hidden states {b.total_len * cfg.d * 2 / 1e9:.1f} GB, "
                          f"W {cfg.V * cfg.d * 2 / 1e9:.2f} GB, dZ chunk {args.chunk_rows * cfg.V * 2 / 1e9:.1f} GB)",
-                   "parallelism": "replicas" if world > 1 else "single GPU"},
+                   "parallelism": ("data-parallel: prompt shards (global batch = ranks x P prompts, cutoffs "
+                                   "by global completion index), dW and loss all-reduced over NCCL" if dp
+                                   else "replicas" if world > 1 else "single GPU")},
         "pct_bf16_peak": {"credited_6NdV_tflops": credited_tf,
                           "of_measured_cublas_sustained": credited_tf / peak_tf,
                           "of_measured_cublas_burst": credited_tf / peaks["bf16_tflops"],
@@ -386,7 +399,9 @@ def run_ours(args):
                                        f"'measured_cublas' = MEASURED_PEAKS.json (torch.matmul 8192^3)"},
         "per_call_ms": {"sample": float(per[:, 0].mean()), "pack": float(per[:, 1].mean()),
                         "fwd": float(per[:, 2].mean()), "bwd": float(per[:, 3].mean()),
-                        "note": "pack includes its one host synchronisation (reading N)"},
+                        "exchange": float(per[:, 4].mean()),
+                        "note": "pack includes its one host synchronisation (reading N); exchange = the "
+                                "all-reduce of dW and the loss (data-parallel runs only)"},
         "pass_stats": pass_stats,
         "roofline": roofline,
         "roofline_backward": ({"kernels": "recompute + dH + dW GEMMs (executed 6*N*d*V per step)", "bound": "tensor",
@@ -613,6 +628,8 @@ def main():
     ap.add_argument("--ref-rows", type=int, default=32)
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--no-design", action="store_true", help="skip timing the cutoff-design stage")
+    ap.add_argument("--replicas", action="store_true",
+                    help="with several ranks: independent replicas, no exchange of dW")
     args = ap.parse_args()
     if args.warmup < 3 and args.impl == "ours":
         args.warmup = 3

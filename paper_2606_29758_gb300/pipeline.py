@@ -142,6 +142,50 @@ def prompt_shard(P: int, K: int, L, world: int, rank: int) -> PromptShard:
     return PromptShard(p0, p1, k0, k1, o0, o0 + sum(lens[k0:k1]))
 
 
+class DataParallelUpdate:
+    """One rank's step of a data-parallel update: its prompt shard through an update pass, then the
+    sum of dW and of the loss over the ranks of a process group.
+
+    The pass must have been built with the global loss scale 1/(P K) of the whole batch, and
+    `traj_base` is the global index of the shard's first completion (PromptShard.k0, or rank * B
+    when every rank holds B completions), so that each completion draws the cutoff it draws in the
+    whole batch. The summed dW and loss are then the whole batch's (Eq. full_update_G and Eq.
+    truncated_update_Ghat: 1/K per prompt, the mean over all prompts). The exchange is one
+    all-reduce of dW (V x d f32) and one of the loss, enqueued on the current stream after the
+    backward; with one rank, or no initialised process group, there is nothing to exchange.
+    `update_pass` needs sample / pack / forward / backward and the tensors dW and loss (UpdatePass).
+    """
+
+    def __init__(self, update_pass, traj_base: int, group=None):
+        self.up = update_pass
+        self.traj_base = int(traj_base)
+        self.group = group
+
+    def world(self) -> int:
+        import torch.distributed as dist
+        if not (dist.is_available() and dist.is_initialized()):
+            return 1
+        return dist.get_world_size(self.group)
+
+    def exchange(self):
+        """Sum dW and the loss over the ranks."""
+        if self.world() > 1:
+            import torch.distributed as dist
+            dist.all_reduce(self.up.dW, group=self.group)
+            dist.all_reduce(self.up.loss, group=self.group)
+
+    def run(self, q, L, R, tok_full, oldlogp_full, hid_full, W, seed, step) -> int:
+        """Sample, pack, forward and backward on this rank's shard, then the exchange; returns the
+        shard's packed rows."""
+        up = self.up
+        up.sample(q, L, seed, step, traj_base=self.traj_base)
+        n = up.pack(L, R, tok_full, oldlogp_full, hid_full)
+        up.forward(W)
+        up.backward(W)
+        self.exchange()
+        return n
+
+
 class InputStager:
     """Double-buffered host -> device staging of the unpacked batch inputs.
 
