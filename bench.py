@@ -487,8 +487,9 @@ def _oracle_head(cfg, b, W64, pk, rows):
 def _oracle_timing(cfg, b, W64, rows, step):
     """One step of the oracle, timed in two parts: the whole batch's cutoffs, advantages and packing
     indices (in full), and the head over a sample of `rows` packed rows. The head's work is linear in
-    the rows (each row's forward and dH; dW sums row by row), so a whole step's time is the prefix
-    time plus N times the head's per-row time."""
+    the rows (each row's forward and dH; dW sums block by block of 128 rows, each block touching all
+    of V x d, so a sample of whole blocks costs per row what a whole step does), so a whole step's
+    time is the prefix time plus N times the head's per-row time."""
     t0 = time.perf_counter()
     pk = _oracle_prefix(cfg, b, step)
     t1 = time.perf_counter()
@@ -625,7 +626,9 @@ def main():
     ap.add_argument("--config", default=WORKLOAD)
     ap.add_argument("--chunk-rows", type=int, default=65536)
     ap.add_argument("--cpu-rows", type=int, default=256)
-    ap.add_argument("--ref-rows", type=int, default=32)
+    # whole 128-row blocks of the oracle's head (its dW update touches all of V x d once per block),
+    # so that the per-row cost of the sample is the per-row cost of a whole step
+    ap.add_argument("--ref-rows", type=int, default=128)
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--no-design", action="store_true", help="skip timing the cutoff-design stage")
     ap.add_argument("--replicas", action="store_true",
