@@ -7,7 +7,8 @@ truncated_update_Ghat), compared element by element and within 1e-3 relative. On
 batches it evaluates a stratified set of rows that touches every 128-row block and both sides
 of every place where the launch schedule changes hands (forward bands, backward chunks,
 recompute and dH/dW bands, the last partial tile), plus every row where the clip binds and the
-largest weights. dH is compared on that set on every batch. For dW, which sums over every row,
+largest weights (or on every row, when the environment variable PSPPO_EVERY_ROW names the
+workload). dH is compared on that set on every batch. For dW, which sums over every row,
 two properties that hold at any size are checked: sum_v dW[v, :] = 0 (the softmax score e_o - p
 sums to zero over the vocabulary) within the bound set by the bf16 rounding of dZ, and
 loss = sum of row losses. Then dW itself: the backward runs again over all N rows of the
@@ -15,6 +16,8 @@ oracle's packed batch with the oracle's lse and coef on the stratified rows and 
 every other row (whose dZ row is then zero), so dW = sum over those rows, which the oracle
 evaluates on every vocabulary row that one of them chose plus 512 random ones.
 """
+import os
+
 import numpy as np
 import pytest
 import torch
@@ -68,7 +71,8 @@ def test_full_size(name):
     heavy = np.argsort(pk["w"])[-16:]
     rows = np.unique(np.concatenate([schedule_rows(cfg, N, CHUNK), bind, heavy])).astype(np.int64)
     assert np.unique(rows // 128).size == -(-N // 128)          # every 128-row block is touched
-    every_row = name == "1.5b"
+    # every row on 1.5B; others on request (PSPPO_EVERY_ROW=7b,long: the oracle then takes minutes)
+    every_row = name == "1.5b" or name in os.environ.get("PSPPO_EVERY_ROW", "").split(",")
     fwd_rows = np.arange(N) if every_row else rows
     res = oracle_rows(cfg, b.W, pk["hid"][fwd_rows], pk["tok"][fwd_rows], pk["oldlogp"][fwd_rows],
                       pk["adv"][fwd_rows], pk["w"][fwd_rows], dh_mask=np.isin(fwd_rows, rows))
