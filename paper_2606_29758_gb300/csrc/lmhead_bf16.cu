@@ -527,7 +527,7 @@ int fwd_gemm_bf16(int64_t N, int d, int V, const void* Hpk, const void* W, const
 // blocks, whose column tiles run side by side, so each panel of dZ (the large operand) is read
 // from DRAM about once and the small operand once per wave (measured on the 7B-shaped step:
 // bands of 4 beat 1, 2, 8 and 16 by 0.3-1.8% of the backward).
-constexpr int kBandRecompute = 48;
+constexpr int kBandRecompute = 32;
 constexpr int kBandGrad = 4;
 
 int proxy_gemm_bf16(int64_t N, int d, int V, const void* Hrows, const void* W, const int32_t* tok, float4* part,

@@ -193,23 +193,57 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
           if (!mbar_wait(&sm.tempty[acc], aph ^ 1u, timeout_ns, abort)) { ok = false; break; }
           tc_fence_after();
           const uint32_t d_tmem = tmem_base + acc * kBN;  // NB = 1: halves at columns 0 and 256
-          for (int kb = 0; kb < sched.num_kb; ++kb, ++kc) {
-            const int s = kc % S;
-            const uint32_t ph = (kc / S) & 1u;
-            if (!mbar_wait(&sm.full[s], ph, timeout_ns, abort)) { ok = false; break; }
-            tc_fence_after();
+          // the MMAs of half h of k-block kb, from stage s (each half accumulates in k order)
+          auto issue_half = [&](int h, int s, int kb) {
             const uint32_t a_base = smem_addr(sm.a[s]);
             const uint32_t b_base = smem_addr(sm.b[s]);
 #pragma unroll
             for (int k = 0; k < kBK / 16; ++k) {
               const uint64_t bd = smem_desc_sw128(b_base + k * b_step, b_lbo, 1024);
-#pragma unroll
-              for (int h = 0; h < HALVES; ++h) {
-                const uint64_t ad = smem_desc_sw128(a_base + h * kTileABytes + k * a_step, a_lbo, 1024);
-                umma_bf16(d_tmem + h * kBN, ad, bd, idesc, (kb | k) != 0 ? 1u : 0u);
+              const uint64_t ad = smem_desc_sw128(a_base + h * kTileABytes + k * a_step, a_lbo, 1024);
+              umma_bf16(d_tmem + h * kBN, ad, bd, idesc, (kb | k) != 0 ? 1u : 0u);
+            }
+          };
+          if constexpr (HALVES == 1) {
+            for (int kb = 0; kb < sched.num_kb; ++kb, ++kc) {
+              const int s = kc % S;
+              const uint32_t ph = (kc / S) & 1u;
+              if (!mbar_wait(&sm.full[s], ph, timeout_ns, abort)) { ok = false; break; }
+              tc_fence_after();
+              issue_half(0, s, kb);
+              umma_commit(&sm.empty[s]);  // frees the stage once these MMAs have read it
+            }
+          } else {
+            // A wide tile's two halves own TMEM columns [0, 256) and [256, 512), and the epilogue
+            // hands each back as soon as it has read it (tempty[0], then tempty[1]). The tile starts
+            // once half 0 is free; while the epilogue still reads half 1 of the previous tile, the
+            // leading k-blocks run on half 0 only and keep their stages; their half-1 MMAs follow, in
+            // k order, as soon as half 1 is free -- at the latest when every stage is held.
+            bool h1_free = false;
+            const uint32_t kc0 = kc;
+            for (int kb = 0; kb < sched.num_kb; ++kb, ++kc) {
+              const int s = kc % S;
+              const uint32_t ph = (kc / S) & 1u;
+              if (!mbar_wait(&sm.full[s], ph, timeout_ns, abort)) { ok = false; break; }
+              tc_fence_after();
+              issue_half(0, s, kb);
+              if (h1_free) {
+                issue_half(1, s, kb);
+                umma_commit(&sm.empty[s]);
+                continue;
+              }
+              if (!mbar_try_wait(&sm.tempty[1], aph ^ 1u)) {
+                if (kb + 1 < S && kb + 1 < sched.num_kb) continue;   // a stage is left: run ahead on half 0
+                if (!mbar_wait(&sm.tempty[1], aph ^ 1u, timeout_ns, abort)) { ok = false; break; }
+              }
+              h1_free = true;
+              tc_fence_after();
+              for (int j = 0; j <= kb; ++j) {          // the held k-blocks' half 1, in order
+                const int sj = (kc0 + j) % S;
+                issue_half(1, sj, j);
+                umma_commit(&sm.empty[sj]);
               }
             }
-            umma_commit(&sm.empty[s]);  // frees the stage once these MMAs have read it
           }
           if (ok) umma_commit(&sm.tfull[acc]);  // accumulator ready for the epilogue
         }
@@ -254,10 +288,11 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
             uint32_t r[32];
             tmem_ld32(t_row + c * 32, r);
             tmem_ld_wait();
-            if (h == HALVES - 1 && c == kBN / 32 - 1) {
-              // the accumulator has been read completely: hand it back to the MMA warp
+            if (c == kBN / 32 - 1) {
+              // this half of the accumulator has been read: hand it back to the MMA warp (a wide
+              // tile returns its two halves one after the other, tempty[0] and tempty[1])
               tc_fence_before();
-              mbar_arrive(&sm.tempty[acc]);
+              mbar_arrive(&sm.tempty[HALVES == 2 ? h : acc]);
             }
             const int col0 = nb * kBN + c * 32;
             if constexpr (Epi::kTmaStore) {
