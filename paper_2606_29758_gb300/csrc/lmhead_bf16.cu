@@ -522,8 +522,9 @@ int fwd_gemm_bf16(int64_t N, int d, int V, const void* Hpk, const void* W, const
   return launch_gemm_single<false, false, FwdLseEpi, 2>(ta, tb, ta, N, V, d, splits, band, ep, status, s);
 }
 
-// Bands (row blocks walked together) of the backward GEMMs. Recompute: 48 row blocks share
-// each W tile (their hidden rows, 44 MB at d = 3584, stay in L2). dH and dW: bands of 4 row
+// Bands (row blocks walked together) of the backward GEMMs. Recompute: 32 row blocks of 128 rows
+// (16 of its 256-row tiles) share each W tile; their hidden rows, 29 MB at d = 3584, stay in L2
+// beside the W tiles in flight and the streamed dZ (44 MB bands read 46% more DRAM). dH and dW: bands of 4 row
 // blocks, whose column tiles run side by side, so each panel of dZ (the large operand) is read
 // from DRAM about once and the small operand once per wave (measured on the 7B-shaped step:
 // bands of 4 beat 1, 2, 8 and 16 by 0.3-1.8% of the backward).
