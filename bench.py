@@ -40,9 +40,9 @@ MEASURED_PEAKS = os.path.join(ROOT, "MEASURED_PEAKS.json")
 FALLBACK_PEAKS = {"hbm_gbs": 6800.0, "bf16_tflops": 1900.0, "bf16_tflops_sustained": 1700.0}
 
 # DRAM bytes (read + write) per launch of the forward GEMM on the 7b workload, the mean of the
-# six launches in profiles/lmhead_pass_7b_launch_list.md (53.25 GB read + 0.92 GB written).
+# six launches in profiles/lmhead_pass_7b_launch_list.md (53.15 GB read + 0.92 GB written).
 # Reset to None whenever the forward kernel or its schedule changes.
-FWD_GEMM_TRAFFIC = {"7b": 54.17e9}
+FWD_GEMM_TRAFFIC = {"7b": 54.07e9}
 
 
 def describe(cfg) -> str:
