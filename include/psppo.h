@@ -147,6 +147,11 @@ int ps_pack_prefixes(int P, int K, int T_max, int d, int dtype,
  *   coef_i = d loss / d logp_i = -loss_scale * w_i * adv_i * ratio_i, or 0 where the
  *   clip binds ((adv > 0 and ratio > 1+eps) or (adv < 0 and ratio < 1-eps)).
  * loss_scale is 1/(P*K) for the paper's estimator (1/K per prompt, mean over prompts).
+ * Data-parallel use: split the batch by whole prompt groups (advantages are per group),
+ * give every shard's ps_sample_cutoffs the global index of its first completion as
+ * traj_base and every shard's forward the whole batch's 1/(P*K); the sums of the shards'
+ * losses and dW (an all-reduce across devices, or PS_DW_ACCUMULATE for shards run one
+ * after another on one device) are then the whole batch's (Eq. full_update_G).
  *
  * Hpk [N][d], W [V][d]: dtype PS_DTYPE_BF16 (tcgen05 tensor cores) or PS_DTYPE_F32
  * (f32 CUDA cores). tok [N] int32 (0 <= tok < V, else PS_DEV_BAD_TOKEN), oldlogp,
