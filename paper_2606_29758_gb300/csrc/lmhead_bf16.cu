@@ -479,9 +479,10 @@ constexpr uint32_t kBRowsBox = kBN;
 // backward 381.4 vs 382.8 ms, and 387.7 ms with per-thread stores of 128-row tiles, back to back).
 constexpr int kRecHalves = 2;
 // The forward's (and score proxy's) tile height depends on the hidden size: its K loop is d long,
-// while the epilogue of a wide tile is a fixed cost that is not overlapped. Measured back to back:
-// at d = 3584 the wide tile is 1% faster, at d = 1536 the 128-row tile is 7% faster.
-static int fwd_halves(int d) { return d < 2560 ? 1 : 2; }
+// while the epilogue of a wide tile overlaps the next tile only in part (one TMEM half at a time).
+// Measured back to back with the current epilogue: at d = 1536 the wide tile is 3% faster (56.5 vs
+// 58.2 ms per 191k-row forward); below d = 1024 the K loop is short enough to keep 128-row tiles.
+static int fwd_halves(int d) { return d < 1024 ? 1 : 2; }
 
 // The forward keeps one band of row blocks in flight; every CTA re-reads its row block for
 // every vocabulary tile, so the band's hidden rows must stay in L2 (129 MB) next to the W

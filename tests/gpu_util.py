@@ -110,7 +110,7 @@ def schedule_rows(cfg, N, ws_chunk_rows, seed=1234):
     def edge(e):
         rows.update(r for r in (e - 1, e) if 0 <= r < N)
 
-    tile = 128 * (2 if cfg.d >= 2560 else 1)          # the forward's tile height at this d
+    tile = 128 * (2 if cfg.d >= 1024 else 1)          # the forward's tile height at this d
     band = max(1, int(FWD_BAND_L2_BYTES // (tile * cfg.d * 2)))
     for e in range(0, N, band * tile):
         edge(e)
