@@ -3,15 +3,15 @@
 //   D[M, N] = sum_k A[m, k] B[n, k]      (bf16 operands, f32 accumulation in TMEM)
 //
 // A is K-major ([M][K] in memory) or MN-major ([K][M]); likewise B ([N][K] or [K][N]).
-// Tiles of 128 x 256 outputs, 64-deep K blocks, 4-stage shared-memory ring fed by TMA
-// with 128-byte swizzle. Roles (192 threads):
+// Tiles of 128 x 256 or 256 x 256 outputs (HALVES, below), 64-deep K blocks, a shared-memory
+// ring fed by TMA with 128-byte swizzle. Roles (192 threads):
 //   warp 0      TMA producer (one lane)
 //   warp 1      TMEM allocator + MMA issuer (one lane)
 //   warps 2..5  epilogue: each thread owns one accumulator row (TMEM lane) and reads
 //               its 256 columns in chunks of 32 with tcgen05.ld
-// Two 256-column accumulators (all 512 TMEM columns) let the epilogue of one tile
-// overlap the main loop of the next. Every wait is bounded; on expiry the kernel sets
-// PS_DEV_TIMEOUT, waits (bounded) for its own loads in flight, frees TMEM and returns.
+// An epilogue either stores from registers itself or (Epi::kTmaStore) stages 32 x 32 slices in
+// shared memory for TMA tensor stores through a third map. Every wait is bounded; on expiry the
+// kernel sets PS_DEV_TIMEOUT, waits (bounded) for its own loads in flight, frees TMEM and returns.
 //
 // Work is split into units: unit u is (m block, range of n blocks [n0, n1)), walked in
 // order by one CTA, so an epilogue can keep per-row state across a unit's tiles (the
@@ -55,11 +55,13 @@ struct Sched {
   }
 };
 
-// HALVES = 1: 128 x 256 tiles, two TMEM accumulators (double-buffered), 4-stage 48 KB ring.
+// HALVES = 1: 128 x 256 tiles, two TMEM accumulators (double-buffered, all 512 columns), so the
+// epilogue of one tile overlaps the main loop of the next; 4-stage 48 KB ring.
 // HALVES = 2: 256 x 256 tiles computed as two M = 128 MMAs that share each B stage, one
-// accumulator pair filling TMEM (not double-buffered), 3-stage 64 KB ring. The wide tile reads
-// a third fewer operand bytes per FLOP; the epilogue of a tile is not overlapped with the next
-// tile's main loop. Each epilogue thread owns one row of each half (two epilogue states).
+// accumulator pair filling TMEM, 3-stage 64 KB ring. The wide tile reads a third fewer operand
+// bytes per FLOP. Its epilogue hands TMEM back half by half and the next tile runs ahead on the
+// first half for as many k-blocks as the ring holds, so the epilogue overlaps the next tile only
+// in part. Each epilogue thread owns one row of each half (two epilogue states).
 template <int HALVES>
 struct GemmCfg {
   static constexpr int kStagesH = HALVES == 1 ? 4 : 3;
