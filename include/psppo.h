@@ -51,7 +51,9 @@ typedef enum {
 enum { PS_MODE_TRUNC = 0, PS_MODE_FULL = 1, PS_MODE_TRUNC_ZERO = 2 };
 enum { PS_DTYPE_BF16 = 0, PS_DTYPE_F32 = 1 };
 enum { PS_ADV_CENTERED = 0, PS_ADV_GROUP_NORM = 1 };
-enum { PS_DW_OVERWRITE = 0, PS_DW_ACCUMULATE = 1 };
+/* Backward flags (bits): dW overwritten (0) or added to (PS_DW_ACCUMULATE); dH likewise
+ * (PS_DH_ACCUMULATE, e.g. to sum the terms of vocabulary shards run on one device). */
+enum { PS_DW_OVERWRITE = 0, PS_DW_ACCUMULATE = 1, PS_DH_ACCUMULATE = 2 };
 
 /* Device status bits (the word at offset 0 of every workspace). */
 enum {
@@ -179,7 +181,7 @@ int ps_lmhead_ppo_fwd(int64_t N, int d, int V, int dtype, const void* Hpk, const
  *
  * Appendix D: d logp / dz = e_o - p. With coef from the forward:
  *   dZ_iv = coef_i (1[v = tok_i] - exp(z_iv - lse_i)),
- *   dH = dZ W            [N][d] f32 (overwritten),
+ *   dH = dZ W            [N][d] f32 (overwritten, or added to with PS_DH_ACCUMULATE),
  *   dW = dZ^T Hpk        [V][d] f32 (overwritten, or added to with PS_DW_ACCUMULATE).
  * The logits are recomputed tile by tile; dZ is held, in the operand dtype, only
  * for one chunk of rows at a time inside the workspace: the rows are split into as
@@ -194,6 +196,56 @@ int ps_lmhead_ppo_bwd(int64_t N, int d, int V, int dtype, const void* Hpk, const
                       const int32_t* tok, const float* lse, const float* coef,
                       float* dH, float* dW, int flags,
                       void* ws, size_t ws_bytes, ps_stream_t stream);
+
+/* ---------------------------------------------------------------------------
+ * Vocabulary-parallel head: W split by vocabulary rows across devices.
+ *
+ * The same loss and gradients as ps_lmhead_ppo_fwd / ps_lmhead_ppo_bwd (Eq. 1 through
+ * the head of Appendix D) when each device holds a shard W_shard = rows [v0, v0 + Vs)
+ * of W [V][d] and every packed row. Per step:
+ *   1. every shard: ps_lmhead_logit_stats -> its per-row statistics (12 bytes a row);
+ *   2. gather the S shards' statistics on every device ([S][N] each, shard order);
+ *   3. every device: ps_lmhead_ppo_fwd_from_stats -> loss, lse, logp, ratio, coef,
+ *      row_loss, identical on all devices;
+ *   4. every shard: ps_lmhead_ppo_bwd_vocab_shard -> its dW rows and its part of dH;
+ *   5. sum the S parts of dH.
+ * The steps run on one device too, shard after shard (a head larger than one launch
+ * should take, or a test of the split).
+ *
+ * ps_lmhead_logit_stats: for every row i, with z_iv = W[v] . Hpk[i] over the shard,
+ *   stats[i] = (m_i, s_i), m_i = max_v z_iv log2(e), s_i = sum_v 2^(z_iv log2(e) - m_i),
+ *   ztok[i]  = z_{i, tok_i} if v0 <= tok_i < v0 + Vs, else -inf.
+ *   stats is [N][2] f32 (8-byte aligned), ztok [N] f32; tok holds global token ids and
+ *   is not range-checked here (a shard does not know the others' range).
+ *   ws_bytes >= ps_lmhead_logit_stats_workspace_size(N, d, Vs, dtype); fewer bytes
+ *   than that give fewer vocabulary ranges, as for the forward.
+ * ps_lmhead_ppo_fwd_from_stats: stats [S][ld][2] and ztok [S][ld] of the S shards (ld >= N
+ *   rows between shards; rows [0, N) of each are read); per
+ *   row, m = max_r m_r, s = sum_r s_r 2^(m_r - m), lse = (m + log2 s) ln 2, the chosen
+ *   logit from the shard that holds it, then the forward's outputs exactly as defined
+ *   under ps_lmhead_ppo_fwd (a token id outside [0, V) sets PS_DEV_BAD_TOKEN and gives
+ *   NaN in its row and the loss). ws_bytes >= ps_lmhead_ppo_fwd_from_stats_workspace_size(N).
+ * ps_lmhead_ppo_bwd_vocab_shard: ps_lmhead_ppo_bwd over the shard, with global token ids
+ *   (the one-hot term applies where tok_i - v0 is in [0, Vs)) and the lse and coef of
+ *   step 3: dW_shard [Vs][d] is the shard's rows of dW; dH [N][d] is the shard's term of
+ *   dH (the S terms sum to dH; with PS_DH_ACCUMULATE it is added to dH, which sums the
+ *   shards run one after another on one device). Requires 0 <= v0, v0 + Vs <= V; workspace as for
+ *   ps_lmhead_ppo_bwd_workspace_size(N, d, Vs, dtype, chunk_rows).
+ * ------------------------------------------------------------------------- */
+size_t ps_lmhead_logit_stats_workspace_size(int64_t N, int d, int Vs, int dtype);
+int ps_lmhead_logit_stats(int64_t N, int d, int Vs, int64_t v0, int dtype, const void* Hpk,
+                          const void* W_shard, const int32_t* tok, float* stats, float* ztok,
+                          void* ws, size_t ws_bytes, ps_stream_t stream);
+size_t ps_lmhead_ppo_fwd_from_stats_workspace_size(int64_t N);
+int ps_lmhead_ppo_fwd_from_stats(int64_t N, int S, int64_t ld, int V, const float* stats, const float* ztok,
+                                 const int32_t* tok, const float* oldlogp, const float* adv,
+                                 const float* w, double eps, double loss_scale, double* loss,
+                                 float* lse, float* logp, float* ratio, float* coef,
+                                 float* row_loss, void* ws, size_t ws_bytes, ps_stream_t stream);
+int ps_lmhead_ppo_bwd_vocab_shard(int64_t N, int d, int Vs, int64_t v0, int V, int dtype,
+                                  const void* Hpk, const void* W_shard, const int32_t* tok,
+                                  const float* lse, const float* coef, float* dH, float* dW_shard,
+                                  int flags, void* ws, size_t ws_bytes, ps_stream_t stream);
 
 /* ---------------------------------------------------------------------------
  * ps_lmhead_score_proxy -- per-token output-head score proxy (cutoff design input).

@@ -19,7 +19,7 @@ PS_OK, PS_ERR_INVALID_ARG, PS_ERR_UNSUPPORTED, PS_ERR_WORKSPACE, PS_ERR_CAPACITY
 PS_MODE_TRUNC, PS_MODE_FULL, PS_MODE_TRUNC_ZERO = 0, 1, 2
 PS_DTYPE_BF16, PS_DTYPE_F32 = 0, 1
 PS_ADV_CENTERED, PS_ADV_GROUP_NORM = 0, 1
-PS_DW_OVERWRITE, PS_DW_ACCUMULATE = 0, 1
+PS_DW_OVERWRITE, PS_DW_ACCUMULATE, PS_DH_ACCUMULATE = 0, 1, 2
 PS_DEV_BAD_PMF, PS_DEV_BAD_LENGTH, PS_DEV_CAPACITY, PS_DEV_BAD_TOKEN, PS_DEV_TIMEOUT, PS_DEV_NONFINITE = \
     1, 2, 4, 8, 16, 32
 
@@ -29,6 +29,8 @@ EXPORTS = [
     "ps_pack_prefixes_workspace_size", "ps_pack_prefixes",
     "ps_lmhead_ppo_fwd_workspace_size", "ps_lmhead_ppo_fwd",
     "ps_lmhead_ppo_bwd_workspace_size", "ps_lmhead_ppo_bwd",
+    "ps_lmhead_logit_stats_workspace_size", "ps_lmhead_logit_stats",
+    "ps_lmhead_ppo_fwd_from_stats_workspace_size", "ps_lmhead_ppo_fwd_from_stats", "ps_lmhead_ppo_bwd_vocab_shard",
     "ps_diag_gemm_bf16", "ps_diag_wait_timeout", "ps_lmhead_ppo_fwd_noalloc",
     "ps_lmhead_score_proxy_workspace_size", "ps_lmhead_score_proxy",
     "ps_design_cutoffs_workspace_size", "ps_design_cutoffs",
@@ -42,7 +44,7 @@ __all__ = EXPORTS + [
     "PS_OK", "PS_ERR_INVALID_ARG", "PS_ERR_UNSUPPORTED", "PS_ERR_WORKSPACE", "PS_ERR_CAPACITY",
     "PS_ERR_DEVICE_DATA", "PS_ERR_TIMEOUT", "PS_ERR_CUDA", "PS_MODE_TRUNC", "PS_MODE_FULL", "PS_MODE_TRUNC_ZERO",
     "PS_DTYPE_BF16", "PS_DTYPE_F32", "PS_ADV_CENTERED", "PS_ADV_GROUP_NORM", "PS_DW_OVERWRITE",
-    "PS_DW_ACCUMULATE", "PS_DEV_BAD_PMF", "PS_DEV_BAD_LENGTH", "PS_DEV_CAPACITY", "PS_DEV_BAD_TOKEN",
+    "PS_DW_ACCUMULATE", "PS_DH_ACCUMULATE", "PS_DEV_BAD_PMF", "PS_DEV_BAD_LENGTH", "PS_DEV_CAPACITY", "PS_DEV_BAD_TOKEN",
     "PS_DEV_TIMEOUT", "PS_DEV_NONFINITE", "PS_DESIGN_OPTIMIZED", "PS_DESIGN_HEURISTIC", "PS_DESIGN_UNIFORM",
     "PS_DESIGN_TIME_PRIOR", "PS_DESIGN_FIXED",
 ]
@@ -74,6 +76,13 @@ _SIGS = {
                                  _vp, _vp, _vp, _vp, _vp, _vp, _vp, _sz, _vp]),
     "ps_lmhead_ppo_bwd_workspace_size": (_sz, [_i64, _i32, _i32, _i32, _i64]),
     "ps_lmhead_ppo_bwd": (_i32, [_i64, _i32, _i32, _i32, _vp, _vp, _vp, _vp, _vp, _vp, _vp, _i32, _vp, _sz, _vp]),
+    "ps_lmhead_logit_stats_workspace_size": (_sz, [_i64, _i32, _i32, _i32]),
+    "ps_lmhead_logit_stats": (_i32, [_i64, _i32, _i32, _i64, _i32, _vp, _vp, _vp, _vp, _vp, _vp, _sz, _vp]),
+    "ps_lmhead_ppo_fwd_from_stats_workspace_size": (_sz, [_i64]),
+    "ps_lmhead_ppo_fwd_from_stats": (_i32, [_i64, _i32, _i64, _i32, _vp, _vp, _vp, _vp, _vp, _vp, _f64, _f64, _vp, _vp,
+                                            _vp, _vp, _vp, _vp, _vp, _sz, _vp]),
+    "ps_lmhead_ppo_bwd_vocab_shard": (_i32, [_i64, _i32, _i32, _i64, _i32, _i32, _vp, _vp, _vp, _vp, _vp, _vp, _vp,
+                                             _i32, _vp, _sz, _vp]),
     "ps_diag_gemm_bf16": (_i32, [_i32, _i32, _i32, _i32, _i32, _vp, _i64, _vp, _i64, _vp, _i64, _i32, _i32, _vp, _sz,
                                  _vp]),
     "ps_diag_wait_timeout": (_i32, [_u64, _vp, _sz, _vp]),
@@ -250,6 +259,37 @@ def ps_lmhead_ppo_bwd(N, d, V, dtype, Hpk, W, tok, lse, coef, dH, dW, flags, ws,
     rc = lib().ps_lmhead_ppo_bwd(N, d, V, dtype, _ptr(Hpk), _ptr(W), _ptr(tok), _ptr(lse), _ptr(coef), _ptr(dH),
                                  _ptr(dW), flags, _ptr(ws), _nbytes(ws), _stream(stream))
     _check(rc, "ps_lmhead_ppo_bwd")
+
+
+def ps_lmhead_logit_stats_workspace_size(N: int, d: int, Vs: int, dtype: int) -> int:
+    return lib().ps_lmhead_logit_stats_workspace_size(N, d, Vs, dtype)
+
+
+def ps_lmhead_logit_stats(N, d, Vs, v0, dtype, Hpk, W_shard, tok, stats, ztok, ws, stream=None):
+    rc = lib().ps_lmhead_logit_stats(N, d, Vs, v0, dtype, _ptr(Hpk), _ptr(W_shard), _ptr(tok), _ptr(stats),
+                                     _ptr(ztok), _ptr(ws), _nbytes(ws), _stream(stream))
+    _check(rc, "ps_lmhead_logit_stats")
+
+
+def ps_lmhead_ppo_fwd_from_stats_workspace_size(N: int) -> int:
+    return lib().ps_lmhead_ppo_fwd_from_stats_workspace_size(N)
+
+
+def ps_lmhead_ppo_fwd_from_stats(N, S, ld, V, stats, ztok, tok, oldlogp, adv, w, eps, loss_scale, loss, lse, logp,
+                                 ratio, coef, row_loss, ws, stream=None):
+    rc = lib().ps_lmhead_ppo_fwd_from_stats(N, S, ld, V, _ptr(stats), _ptr(ztok), _ptr(tok), _ptr(oldlogp), _ptr(adv),
+                                            _ptr(w), float(eps), float(loss_scale), _ptr(loss), _ptr(lse), _ptr(logp),
+                                            _ptr(ratio), _ptr(coef), _ptr(row_loss), _ptr(ws), _nbytes(ws),
+                                            _stream(stream))
+    _check(rc, "ps_lmhead_ppo_fwd_from_stats")
+
+
+def ps_lmhead_ppo_bwd_vocab_shard(N, d, Vs, v0, V, dtype, Hpk, W_shard, tok, lse, coef, dH, dW_shard, flags, ws,
+                                  stream=None):
+    rc = lib().ps_lmhead_ppo_bwd_vocab_shard(N, d, Vs, v0, V, dtype, _ptr(Hpk), _ptr(W_shard), _ptr(tok), _ptr(lse),
+                                             _ptr(coef), _ptr(dH), _ptr(dW_shard), flags, _ptr(ws), _nbytes(ws),
+                                             _stream(stream))
+    _check(rc, "ps_lmhead_ppo_bwd_vocab_shard")
 
 
 def ps_diag_gemm_bf16(M, N, K, a_mn_major, b_mn_major, A, lda, B, ldb, C, ldc, accumulate, ws, variant=0,

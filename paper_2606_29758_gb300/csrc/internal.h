@@ -10,16 +10,17 @@ int num_sms_current();
 int device_is_sm103();
 
 // Forward GEMM with the online-logsumexp epilogue. part: [splits][N] (max2, sum) pairs
-// (max in log2 units); ztok: [N] chosen-token logit.
+// (max in log2 units); ztok: [N] chosen-token logit, written only for rows whose token id minus
+// tok_base falls in [0, V) (W holding vocabulary rows [tok_base, tok_base + V) of a sharded head).
 int fwd_tile_splits_bf16(int V);   // one partial per 256-column vocabulary tile
 // Vocabulary ranges per row block, at most max_splits (the partials the workspace holds); the
 // score proxy uses the same chooser.
 int choose_fwd_splits_bf16(int64_t N, int d, int V, int num_sms, int max_splits);
 int fwd_gemm_bf16(int64_t N, int d, int V, const void* Hpk, const void* W, const int32_t* tok, float2* part,
-                  float* ztok, int splits, uint32_t* status, cudaStream_t s);
+                  float* ztok, int splits, uint32_t* status, cudaStream_t s, int tok_base = 0);
 int fwd_splits_f32(int V);
 int fwd_gemm_f32(int64_t N, int d, int V, const float* Hpk, const float* W, const int32_t* tok, float2* part,
-                 float* ztok, uint32_t* status, cudaStream_t s);
+                 float* ztok, uint32_t* status, cudaStream_t s, int tok_base = 0);
 
 // Score-proxy GEMM (the forward's schedule): part [splits][N] (max2, s1, s2, 0), ztok [N].
 int proxy_gemm_bf16(int64_t N, int d, int V, const void* Hrows, const void* W, const int32_t* tok, float4* part,
@@ -31,13 +32,15 @@ int proxy_topk_gemm_bf16(int64_t N, int d, int V, const void* Hrows, const void*
                          float4* part, float2* topk, float* ztok, int splits, uint32_t* status, cudaStream_t s);
 
 // Backward for one chunk of rows [0, rc) of already offset pointers: recompute dZ into
-// dz ([rc][ldz], operand dtype), then dH = dZ W and dW (+)= dZ^T Hpk.
+// dz ([rc][ldz], operand dtype), then dH = dZ W and dW (+)= dZ^T Hpk. With tok_base, W holds
+// vocabulary rows [tok_base, tok_base + V) and the one-hot term applies where tok - tok_base is in [0, V);
+// dh_accumulate adds dH to what the buffer holds.
 int bwd_chunk_bf16(int64_t rc, int d, int V, const void* Hpk, const void* W, const int32_t* tok,
                    const float* lse, const float* coef, float* dH, float* dW, int dw_accumulate, void* dz,
-                   int64_t ldz, uint32_t* status, cudaStream_t s);
+                   int64_t ldz, uint32_t* status, cudaStream_t s, int tok_base = 0, int dh_accumulate = 0);
 int bwd_chunk_f32(int64_t rc, int d, int V, const float* Hpk, const float* W, const int32_t* tok,
                   const float* lse, const float* coef, float* dH, float* dW, int dw_accumulate, float* dz,
-                  int64_t ldz, uint32_t* status, cudaStream_t s);
+                  int64_t ldz, uint32_t* status, cudaStream_t s, int tok_base = 0, int dh_accumulate = 0);
 
 // Plain tensor-core GEMM (test hook): C[M][N] (+)= sum_k A(m,k) B(k,n), f32 out. variant: 0 one
 // CTA per 128 x 256 tile, 1 a CTA pair per 256 x 256 tile, 2 one CTA per 256 x 256 tile.

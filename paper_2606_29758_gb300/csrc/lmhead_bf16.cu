@@ -38,6 +38,7 @@ struct FwdLseEpi {
     int M, N;
     float2* part;
     float* ztok;
+    int tok_base;   // token ids are global; W holds vocabulary rows [tok_base, tok_base + N)
   };
   struct State {
     float m2, s;
@@ -46,7 +47,7 @@ struct FwdLseEpi {
   static __device__ __forceinline__ void begin_unit(const Params& p, State& st, int row, int) {
     st.m2 = -INFINITY;
     st.s = 0.f;
-    st.tok = row < p.M ? __ldg(p.tok + row) : -1;
+    st.tok = row < p.M ? __ldg(p.tok + row) - p.tok_base : -1;
   }
   static __device__ __forceinline__ void chunk(const Params& p, State& st, int row, int col0,
                                                const uint32_t (&r)[32]) {
@@ -238,6 +239,7 @@ struct BwdDzEpi {
     const float* lse;
     const float* coef;
     int M, N;
+    int tok_base;   // token ids are global; W holds vocabulary rows [tok_base, tok_base + N)
   };
   struct State {
     float lse2, coef;
@@ -246,7 +248,7 @@ struct BwdDzEpi {
   static __device__ __forceinline__ int cols(const Params& p) { return p.N; }
   static __device__ __forceinline__ void begin_unit(const Params& p, State& st, int row, int) {
     if (row < p.M) {
-      st.tok = __ldg(p.tok + row);
+      st.tok = __ldg(p.tok + row) - p.tok_base;
       st.lse2 = __ldg(p.lse + row) * kLog2e;
       st.coef = __ldg(p.coef + row);
     } else {
@@ -510,12 +512,12 @@ int choose_fwd_splits_bf16(int64_t N, int d, int V, int num_sms, int max_splits)
 }
 
 int fwd_gemm_bf16(int64_t N, int d, int V, const void* Hpk, const void* W, const int32_t* tok, float2* part,
-                  float* ztok, int splits, uint32_t* status, cudaStream_t s) {
+                  float* ztok, int splits, uint32_t* status, cudaStream_t s, int tok_base) {
   const int halves = fwd_halves(d);
   CUtensorMap ta, tb;
   if (!map_kmajor(&ta, Hpk, N, d, d, kBM * halves) || !map_kmajor(&tb, W, V, d, d, kBRowsBox))
     return PS_ERR_INVALID_ARG;
-  FwdLseEpi::Params ep{tok, static_cast<int>(N), V, part, ztok};
+  FwdLseEpi::Params ep{tok, static_cast<int>(N), V, part, ztok, tok_base};
   const int workers = num_sms_current();
   const int band = splits == fwd_tile_splits_bf16(V) ? fwd_band_max(d) : (workers + splits - 1) / splits;
   if (halves == 1)
@@ -561,7 +563,7 @@ int proxy_topk_gemm_bf16(int64_t N, int d, int V, const void* Hrows, const void*
 
 int bwd_chunk_bf16(int64_t rc, int d, int V, const void* Hpk, const void* W, const int32_t* tok,
                    const float* lse, const float* coef, float* dH, float* dW, int dw_accumulate, void* dz,
-                   int64_t ldz, uint32_t* status, cudaStream_t s) {
+                   int64_t ldz, uint32_t* status, cudaStream_t s, int tok_base, int dh_accumulate) {
   int rcode;
   {
     CUtensorMap ta, tb;
@@ -570,7 +572,7 @@ int bwd_chunk_bf16(int64_t rc, int d, int V, const void* Hpk, const void* W, con
     // dZ [rc][ldz] bf16, written in 32 x 32 boxes from 64-byte-swizzled staging
     CUtensorMap tz;
     if (!make_map(&tz, dz, V, rc, ldz * 2, 32, 32, CU_TENSOR_MAP_SWIZZLE_64B)) return PS_ERR_INVALID_ARG;
-    BwdDzEpi::Params ep{tok, lse, coef, static_cast<int>(rc), V};
+    BwdDzEpi::Params ep{tok, lse, coef, static_cast<int>(rc), V, tok_base};
     rcode = launch_gemm_single<false, false, BwdDzEpi, kRecHalves>(ta, tb, tz, rc, V, d, 0,
                                                                     kBandRecompute / kRecHalves, ep, status, s);
     if (rcode != PS_OK) return rcode;
@@ -580,7 +582,7 @@ int bwd_chunk_bf16(int64_t rc, int d, int V, const void* Hpk, const void* W, con
   if (dH) {
     CUtensorMap ta, tb;
     if (!map_kmajor(&ta, dz, rc, V, ldz, 2 * kBM) || !map_mnmajor(&tb, W, V, d, d)) return PS_ERR_INVALID_ARG;
-    StoreF32Epi::Params ep{dH, d, static_cast<int>(rc), d, 0};
+    StoreF32Epi::Params ep{dH, d, static_cast<int>(rc), d, dh_accumulate};
     rcode = launch_gemm_single<false, true, StoreF32Epi, 2>(ta, tb, ta, rc, d, V, 0, kBandGrad, ep, status, s);
     if (rcode != PS_OK) return rcode;
   }

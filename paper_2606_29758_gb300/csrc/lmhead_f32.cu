@@ -68,6 +68,7 @@ struct SimtFwdEpi {
     const int32_t* tok;
     float2* part;   // [n_tiles][M]
     float* ztok;
+    int tok_base;   // token ids are global; W holds vocabulary rows [tok_base, tok_base + N)
   };
   static __device__ __forceinline__ void tile(const Params& p, int64_t M, int64_t N, int64_t r0, int64_t c0,
                                               int ntile, int tx, float (&acc)[4][4]) {
@@ -81,7 +82,7 @@ struct SimtFwdEpi {
         x[j] = (c0 + j < N) ? acc[i][j] * kLog2e : -INFINITY;
         mx = fmaxf(mx, x[j]);
       }
-      const int t = row < M ? __ldg(p.tok + row) : -1;
+      const int t = row < M ? __ldg(p.tok + row) - p.tok_base : -1;
 #pragma unroll
       for (int j = 0; j < 4; ++j)
         if (c0 + j < N && c0 + j == t) p.ztok[row] = acc[i][j];
@@ -104,6 +105,7 @@ struct SimtDzEpi {
     const float* coef;
     float* dz;
     int64_t ldz;
+    int tok_base;
   };
   static __device__ __forceinline__ void tile(const Params& p, int64_t M, int64_t N, int64_t r0, int64_t c0, int,
                                               int, float (&acc)[4][4]) {
@@ -111,7 +113,7 @@ struct SimtDzEpi {
     for (int i = 0; i < 4; ++i) {
       const int64_t row = r0 + i;
       if (row >= M) continue;
-      const int t = __ldg(p.tok + row);
+      const int t = __ldg(p.tok + row) - p.tok_base;
       const float l = __ldg(p.lse + row), c = __ldg(p.coef + row);
 #pragma unroll
       for (int j = 0; j < 4; ++j) {
@@ -161,20 +163,20 @@ static int launch_simt(int64_t M, int64_t N, int64_t K, Operand A, Operand B, co
 int fwd_splits_f32(int V) { return (V + kSB - 1) / kSB; }
 
 int fwd_gemm_f32(int64_t N, int d, int V, const float* Hpk, const float* W, const int32_t* tok, float2* part,
-                 float* ztok, uint32_t*, cudaStream_t s) {
+                 float* ztok, uint32_t*, cudaStream_t s, int tok_base) {
   Operand A{Hpk, d, 1};  // A(m, k) = H[m][k]
   Operand B{W, 1, d};    // B(k, n) = W[n][k]
-  return launch_simt<SimtFwdEpi>(N, V, d, A, B, SimtFwdEpi::Params{tok, part, ztok}, s);
+  return launch_simt<SimtFwdEpi>(N, V, d, A, B, SimtFwdEpi::Params{tok, part, ztok, tok_base}, s);
 }
 
 int bwd_chunk_f32(int64_t rc, int d, int V, const float* Hpk, const float* W, const int32_t* tok,
                   const float* lse, const float* coef, float* dH, float* dW, int dw_accumulate, float* dz,
-                  int64_t ldz, uint32_t*, cudaStream_t s) {
+                  int64_t ldz, uint32_t*, cudaStream_t s, int tok_base, int dh_accumulate) {
   int r = launch_simt<SimtDzEpi>(rc, V, d, Operand{Hpk, d, 1}, Operand{W, 1, d},
-                                 SimtDzEpi::Params{tok, lse, coef, dz, ldz}, s);
+                                 SimtDzEpi::Params{tok, lse, coef, dz, ldz, tok_base}, s);
   if (r != PS_OK) return r;
   if (dH) {  // dH(m=i, n=c) = sum_v dz[i][v] W[v][c]
-    r = launch_simt<SimtStoreEpi>(rc, d, V, Operand{dz, ldz, 1}, Operand{W, d, 1}, SimtStoreEpi::Params{dH, d, 0},
+    r = launch_simt<SimtStoreEpi>(rc, d, V, Operand{dz, ldz, 1}, Operand{W, d, 1}, SimtStoreEpi::Params{dH, d, dh_accumulate},
                                   s);
     if (r != PS_OK) return r;
   }

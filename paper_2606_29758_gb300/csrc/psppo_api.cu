@@ -315,48 +315,56 @@ __global__ void __launch_bounds__(kPackThreads)
 
 // ================================================================== K4: forward finalize
 constexpr int kFinThreads = 256;
-__global__ void __launch_bounds__(kFinThreads)
-    fwd_finalize_kernel(int64_t N, int V, int splits, const float2* __restrict__ part, const float* __restrict__ ztok,
-                        const int32_t* __restrict__ tok, const float* __restrict__ oldlogp,
-                        const float* __restrict__ adv, const float* __restrict__ w, double eps, double loss_scale,
-                        float* __restrict__ lse, float* __restrict__ logp, float* __restrict__ ratio,
-                        float* __restrict__ coef, float* __restrict__ row_loss, double* __restrict__ block_loss,
-                        uint32_t* status) {
-  const int64_t i = static_cast<int64_t>(blockIdx.x) * kFinThreads + threadIdx.x;
-  double rl = 0.0;
-  if (i < N) {
-    float m = -INFINITY;
-    for (int s = 0; s < splits; ++s) m = fmaxf(m, part[static_cast<int64_t>(s) * N + i].x);
-    float S = 0.f;
-    for (int s = 0; s < splits; ++s) {
-      const float2 pr = part[static_cast<int64_t>(s) * N + i];
-      S += pr.y * exp2f(pr.x - m);
-    }
-    const double l = (static_cast<double>(m) + log2(static_cast<double>(S))) * 0.6931471805599453;
-    const int t = tok[i];
-    double lp;
-    if (t < 0 || t >= V) {
-      raise_status(status, PS_DEV_BAD_TOKEN);
-      lp = NAN;
-    } else {
-      lp = static_cast<double>(ztok[i]) - l;
-    }
-    const double r = exp(lp - static_cast<double>(oldlogp[i]));
-    const double A = adv[i], wt = w[i];
-    // min and clip as the definition has them: a NaN ratio (a non-finite input or a bad token
-    // id) gives a NaN surrogate, which fmin / fmax alone would replace by the other operand
-    const double clipped = r != r ? r : fmin(fmax(r, 1.0 - eps), 1.0 + eps);
-    const double ra = r * A, ca = clipped * A;
-    const double sur = (ra != ra || ca != ca) ? NAN : fmin(ra, ca);
-    rl = -loss_scale * wt * sur;
-    const bool bind = (A > 0.0 && r > 1.0 + eps) || (A < 0.0 && r < 1.0 - eps);
-    lse[i] = static_cast<float>(l);
-    logp[i] = static_cast<float>(lp);
-    ratio[i] = static_cast<float>(r);
-    coef[i] = bind ? 0.f : static_cast<float>(-loss_scale * wt * A * r);
-    if (row_loss) row_loss[i] = static_cast<float>(rl);
+
+// One packed row of the forward (Eq. 1 through the head, the loss of Eq. truncated_update_Ghat):
+// from the row's logsumexp in base 2, lse2 = m + log2(S) (m the base-2 maximum, S the sum of
+// 2^(x - m) over the vocabulary), and its chosen logit zt. Returns the row's loss term.
+__device__ __forceinline__ double finalize_row(int64_t i, float m, float S, float zt, int t, int V,
+                                               const float* __restrict__ oldlogp, const float* __restrict__ adv,
+                                               const float* __restrict__ w, double eps, double loss_scale,
+                                               float* __restrict__ lse, float* __restrict__ logp,
+                                               float* __restrict__ ratio, float* __restrict__ coef,
+                                               float* __restrict__ row_loss, uint32_t* status) {
+  const double l = (static_cast<double>(m) + log2(static_cast<double>(S))) * 0.6931471805599453;
+  double lp;
+  if (t < 0 || t >= V) {
+    raise_status(status, PS_DEV_BAD_TOKEN);
+    lp = NAN;
+  } else {
+    lp = static_cast<double>(zt) - l;
   }
-  // fixed-order block sum: warp shuffles, then warp 0 over the warp sums
+  const double r = exp(lp - static_cast<double>(oldlogp[i]));
+  const double A = adv[i], wt = w[i];
+  // min and clip as the definition has them: a NaN ratio (a non-finite input or a bad token
+  // id) gives a NaN surrogate, which fmin / fmax alone would replace by the other operand
+  const double clipped = r != r ? r : fmin(fmax(r, 1.0 - eps), 1.0 + eps);
+  const double ra = r * A, ca = clipped * A;
+  const double sur = (ra != ra || ca != ca) ? NAN : fmin(ra, ca);
+  const double rl = -loss_scale * wt * sur;
+  const bool bind = (A > 0.0 && r > 1.0 + eps) || (A < 0.0 && r < 1.0 - eps);
+  lse[i] = static_cast<float>(l);
+  logp[i] = static_cast<float>(lp);
+  ratio[i] = static_cast<float>(r);
+  coef[i] = bind ? 0.f : static_cast<float>(-loss_scale * wt * A * r);
+  if (row_loss) row_loss[i] = static_cast<float>(rl);
+  return rl;
+}
+
+// The (max, sum) pairs of `count` parts of a row's vocabulary (stride `stride` between parts),
+// merged into one pair: m = max m_s, S = sum S_s 2^(m_s - m).
+__device__ __forceinline__ float2 merge_parts(const float2* __restrict__ part, int count, int64_t stride) {
+  float m = -INFINITY;
+  for (int s = 0; s < count; ++s) m = fmaxf(m, part[static_cast<int64_t>(s) * stride].x);
+  float S = 0.f;
+  for (int s = 0; s < count; ++s) {
+    const float2 pr = part[static_cast<int64_t>(s) * stride];
+    S += pr.y * exp2f(pr.x - m);
+  }
+  return make_float2(m, S);
+}
+
+// Fixed-order block sum of the rows' loss terms: warp shuffles, then warp 0 over the warp sums.
+__device__ __forceinline__ void block_loss_sum(double rl, double* __restrict__ block_loss) {
   __shared__ double ws_sum[kFinThreads / 32];
 #pragma unroll
   for (int o = 16; o >= 1; o >>= 1) rl += __shfl_down_sync(0xffffffffu, rl, o);
@@ -368,6 +376,59 @@ __global__ void __launch_bounds__(kFinThreads)
     for (int o = 16; o >= 1; o >>= 1) v += __shfl_down_sync(0xffffffffu, v, o);
     if (threadIdx.x == 0) block_loss[blockIdx.x] = v;
   }
+}
+
+__global__ void __launch_bounds__(kFinThreads)
+    fwd_finalize_kernel(int64_t N, int V, int splits, const float2* __restrict__ part, const float* __restrict__ ztok,
+                        const int32_t* __restrict__ tok, const float* __restrict__ oldlogp,
+                        const float* __restrict__ adv, const float* __restrict__ w, double eps, double loss_scale,
+                        float* __restrict__ lse, float* __restrict__ logp, float* __restrict__ ratio,
+                        float* __restrict__ coef, float* __restrict__ row_loss, double* __restrict__ block_loss,
+                        uint32_t* status) {
+  const int64_t i = static_cast<int64_t>(blockIdx.x) * kFinThreads + threadIdx.x;
+  double rl = 0.0;
+  if (i < N) {
+    const float2 ms = merge_parts(part + i, splits, N);
+    rl = finalize_row(i, ms.x, ms.y, ztok[i], tok[i], V, oldlogp, adv, w, eps, loss_scale, lse, logp, ratio, coef,
+                      row_loss, status);
+  }
+  block_loss_sum(rl, block_loss);
+}
+
+// A vocabulary shard's statistics: its vocabulary tiles' (max, sum) pairs merged per row, and the
+// chosen logit where the row's token lies in the shard ([tok_base, tok_base + Vs)), -inf elsewhere.
+__global__ void __launch_bounds__(kFinThreads)
+    stats_merge_kernel(int64_t N, int splits, const float2* __restrict__ part, const float* __restrict__ ztok_ws,
+                       const int32_t* __restrict__ tok, int64_t tok_base, int Vs, float2* __restrict__ stats,
+                       float* __restrict__ ztok) {
+  const int64_t i = static_cast<int64_t>(blockIdx.x) * kFinThreads + threadIdx.x;
+  if (i >= N) return;
+  stats[i] = merge_parts(part + i, splits, N);
+  const int64_t t = static_cast<int64_t>(tok[i]) - tok_base;
+  ztok[i] = (t >= 0 && t < Vs) ? ztok_ws[i] : -INFINITY;
+}
+
+// The forward finalize from the statistics of S vocabulary shards ([S][ld] each): their (max, sum)
+// pairs merged as one row's tiles are, and the chosen logit from the shard that holds the token (the
+// largest of the S values, the others being -inf).
+__global__ void __launch_bounds__(kFinThreads)
+    stats_finalize_kernel(int64_t N, int S, int64_t ld, int V, const float2* __restrict__ stats,
+                          const float* __restrict__ ztok,
+                          const int32_t* __restrict__ tok, const float* __restrict__ oldlogp,
+                          const float* __restrict__ adv, const float* __restrict__ w, double eps, double loss_scale,
+                          float* __restrict__ lse, float* __restrict__ logp, float* __restrict__ ratio,
+                          float* __restrict__ coef, float* __restrict__ row_loss, double* __restrict__ block_loss,
+                          uint32_t* status) {
+  const int64_t i = static_cast<int64_t>(blockIdx.x) * kFinThreads + threadIdx.x;
+  double rl = 0.0;
+  if (i < N) {
+    const float2 ms = merge_parts(stats + i, S, ld);
+    float zt = -INFINITY;
+    for (int r = 0; r < S; ++r) zt = fmaxf(zt, ztok[static_cast<int64_t>(r) * ld + i]);
+    rl = finalize_row(i, ms.x, ms.y, zt, tok[i], V, oldlogp, adv, w, eps, loss_scale, lse, logp, ratio, coef,
+                      row_loss, status);
+  }
+  block_loss_sum(rl, block_loss);
 }
 
 __global__ void __launch_bounds__(1024) loss_reduce_kernel(int64_t nblocks, const double* __restrict__ part,
@@ -575,6 +636,70 @@ int ps_lmhead_ppo_fwd(int64_t N, int d, int V, int dtype, const void* Hpk, const
   return cudaGetLastError() == cudaSuccess ? PS_OK : PS_ERR_CUDA;
 }
 
+size_t ps_lmhead_logit_stats_workspace_size(int64_t N, int d, int Vs, int dtype) {
+  return ps_lmhead_ppo_fwd_workspace_size(N, d, Vs, dtype);
+}
+
+int ps_lmhead_logit_stats(int64_t N, int d, int Vs, int64_t v0, int dtype, const void* Hpk, const void* W_shard,
+                          const int32_t* tok, float* stats, float* ztok, void* ws, size_t ws_bytes,
+                          ps_stream_t stream) {
+  NvtxRange nvtx_range("ps_lmhead_logit_stats");
+  if (N < 0 || N > INT32_MAX || Vs < 1 || v0 < 0 || v0 + Vs > INT32_MAX || !dtype_ok(dtype) || !d_ok(d, dtype))
+    return PS_ERR_INVALID_ARG;
+  if (N > 0 && (!Hpk || !W_shard || !tok || !stats || !ztok)) return PS_ERR_INVALID_ARG;
+  if (N > 0 && (!al16(Hpk) || !al16(W_shard) || (reinterpret_cast<uintptr_t>(stats) & 7))) return PS_ERR_INVALID_ARG;
+  if (dtype == PS_DTYPE_BF16 && !device_is_sm103()) return PS_ERR_UNSUPPORTED;
+  cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
+  FwdWs f = fwd_ws(ws, N, Vs, dtype, ws_bytes);
+  if (N > 0 && f.splits < 1) return PS_ERR_WORKSPACE;
+  int rc = begin_call(ws, ws_bytes, f.bytes, s);
+  if (rc != PS_OK || N == 0) return rc;
+  int splits;
+  if (dtype == PS_DTYPE_BF16) {
+    splits = choose_fwd_splits_bf16(N, d, Vs, num_sms_current(), f.splits);
+    rc = fwd_gemm_bf16(N, d, Vs, Hpk, W_shard, tok, f.part, f.ztok, splits, status_word(ws), s, static_cast<int>(v0));
+  } else {
+    splits = fwd_splits_f32(Vs);
+    rc = fwd_gemm_f32(N, d, Vs, static_cast<const float*>(Hpk), static_cast<const float*>(W_shard), tok, f.part,
+                      f.ztok, status_word(ws), s, static_cast<int>(v0));
+  }
+  if (rc != PS_OK) return rc;
+  const int64_t nb = (N + kFinThreads - 1) / kFinThreads;
+  stats_merge_kernel<<<static_cast<unsigned>(nb), kFinThreads, 0, s>>>(N, splits, f.part, f.ztok, tok, v0, Vs,
+                                                                        reinterpret_cast<float2*>(stats), ztok);
+  return cudaGetLastError() == cudaSuccess ? PS_OK : PS_ERR_CUDA;
+}
+
+size_t ps_lmhead_ppo_fwd_from_stats_workspace_size(int64_t N) {
+  if (N < 0) return 0;
+  const int64_t nb = (N + kFinThreads - 1) / kFinThreads;
+  return kWsHeader + align_up(sizeof(double) * static_cast<size_t>(nb > 0 ? nb : 1), 256);
+}
+
+int ps_lmhead_ppo_fwd_from_stats(int64_t N, int S, int64_t ld, int V, const float* stats, const float* ztok,
+                                 const int32_t* tok,
+                                 const float* oldlogp, const float* adv, const float* w, double eps,
+                                 double loss_scale, double* loss, float* lse, float* logp, float* ratio, float* coef,
+                                 float* row_loss, void* ws, size_t ws_bytes, ps_stream_t stream) {
+  NvtxRange nvtx_range("ps_lmhead_ppo_fwd_from_stats");
+  if (N < 0 || N > INT32_MAX || S < 1 || ld < N || V < 1 || !(eps >= 0.0) || !loss) return PS_ERR_INVALID_ARG;
+  if (N > 0 && (!stats || !ztok || !tok || !oldlogp || !adv || !w || !lse || !logp || !ratio || !coef))
+    return PS_ERR_INVALID_ARG;
+  if (N > 0 && (reinterpret_cast<uintptr_t>(stats) & 7)) return PS_ERR_INVALID_ARG;
+  cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
+  int rc = begin_call(ws, ws_bytes, ps_lmhead_ppo_fwd_from_stats_workspace_size(N), s);
+  if (rc != PS_OK) return rc;
+  if (N == 0) return cudaMemsetAsync(loss, 0, sizeof(double), s) == cudaSuccess ? PS_OK : PS_ERR_CUDA;
+  const int64_t nb = (N + kFinThreads - 1) / kFinThreads;
+  double* block_loss = reinterpret_cast<double*>(static_cast<uint8_t*>(ws) + kWsHeader);
+  stats_finalize_kernel<<<static_cast<unsigned>(nb), kFinThreads, 0, s>>>(
+      N, S, ld, V, reinterpret_cast<const float2*>(stats), ztok, tok, oldlogp, adv, w, eps, loss_scale, lse, logp, ratio,
+      coef, row_loss, block_loss, status_word(ws));
+  if (cudaGetLastError() != cudaSuccess) return PS_ERR_CUDA;
+  loss_reduce_kernel<<<1, 1024, 0, s>>>(nb, block_loss, loss);
+  return cudaGetLastError() == cudaSuccess ? PS_OK : PS_ERR_CUDA;
+}
+
 size_t ps_lmhead_ppo_bwd_workspace_size(int64_t N, int d, int V, int dtype, int64_t chunk_rows) {
   if (N < 0 || V < 1 || !dtype_ok(dtype)) return 0;
   (void)d;
@@ -585,12 +710,15 @@ size_t ps_lmhead_ppo_bwd_workspace_size(int64_t N, int d, int V, int dtype, int6
   return kWsHeader + static_cast<size_t>(rows) * ldz_for(V) * elem_size(dtype);
 }
 
-int ps_lmhead_ppo_bwd(int64_t N, int d, int V, int dtype, const void* Hpk, const void* W, const int32_t* tok,
-                      const float* lse, const float* coef, float* dH, float* dW, int flags, void* ws,
-                      size_t ws_bytes, ps_stream_t stream) {
-  NvtxRange nvtx_range("ps_lmhead_ppo_bwd");
+}  // extern "C"
+
+// The backward over a head of V vocabulary rows whose first is global token id tok_base (0 for the
+// whole head, v0 for one shard of a vocabulary-parallel head).
+static int lmhead_bwd_impl(int64_t N, int d, int V, int64_t tok_base, int dtype, const void* Hpk, const void* W,
+                           const int32_t* tok, const float* lse, const float* coef, float* dH, float* dW, int flags,
+                           void* ws, size_t ws_bytes, ps_stream_t stream) {
   if (N < 0 || N > INT32_MAX || V < 1 || !dtype_ok(dtype) || !d_ok(d, dtype)) return PS_ERR_INVALID_ARG;
-  if (flags != PS_DW_OVERWRITE && flags != PS_DW_ACCUMULATE) return PS_ERR_INVALID_ARG;
+  if (flags & ~(PS_DW_ACCUMULATE | PS_DH_ACCUMULATE)) return PS_ERR_INVALID_ARG;
   if (N > 0 && (!Hpk || !W || !tok || !lse || !coef)) return PS_ERR_INVALID_ARG;
   if ((N > 0 && (!al16(Hpk) || !al16(W))) || (dH && !al16(dH)) || (dW && !al16(dW))) return PS_ERR_INVALID_ARG;
   if (dtype == PS_DTYPE_BF16 && !device_is_sm103()) return PS_ERR_UNSUPPORTED;
@@ -598,7 +726,7 @@ int ps_lmhead_ppo_bwd(int64_t N, int d, int V, int dtype, const void* Hpk, const
   int rc = begin_call(ws, ws_bytes, ps_lmhead_ppo_bwd_workspace_size(N, d, V, dtype, 128), s);
   if (rc != PS_OK) return rc;
   if (N == 0) {
-    if (dW && flags == PS_DW_OVERWRITE)
+    if (dW && !(flags & PS_DW_ACCUMULATE))
       return cudaMemsetAsync(dW, 0, sizeof(float) * static_cast<size_t>(V) * d, s) == cudaSuccess ? PS_OK
                                                                                                 : PS_ERR_CUDA;
     return PS_OK;
@@ -615,19 +743,40 @@ int ps_lmhead_ppo_bwd(int64_t N, int d, int V, int dtype, const void* Hpk, const
   void* dz = static_cast<uint8_t*>(ws) + kWsHeader;
   for (int64_t r0 = 0; r0 < N; r0 += chunk) {
     const int64_t rcn = (N - r0) < chunk ? (N - r0) : chunk;
-    const int acc = (r0 > 0 || flags == PS_DW_ACCUMULATE) ? 1 : 0;
+    const int acc = (r0 > 0 || (flags & PS_DW_ACCUMULATE)) ? 1 : 0;
+    const int hacc = (flags & PS_DH_ACCUMULATE) ? 1 : 0;
     if (dtype == PS_DTYPE_BF16) {
       const uint16_t* h = static_cast<const uint16_t*>(Hpk) + r0 * d;
       rc = bwd_chunk_bf16(rcn, d, V, h, W, tok + r0, lse + r0, coef + r0, dH ? dH + r0 * d : nullptr, dW, acc, dz,
-                          ldz, status_word(ws), s);
+                          ldz, status_word(ws), s, static_cast<int>(tok_base), hacc);
     } else {
       const float* h = static_cast<const float*>(Hpk) + r0 * d;
       rc = bwd_chunk_f32(rcn, d, V, h, static_cast<const float*>(W), tok + r0, lse + r0, coef + r0,
-                         dH ? dH + r0 * d : nullptr, dW, acc, static_cast<float*>(dz), ldz, status_word(ws), s);
+                         dH ? dH + r0 * d : nullptr, dW, acc, static_cast<float*>(dz), ldz, status_word(ws), s,
+                         static_cast<int>(tok_base), hacc);
     }
     if (rc != PS_OK) return rc;
   }
   return PS_OK;
+}
+
+extern "C" {
+
+int ps_lmhead_ppo_bwd(int64_t N, int d, int V, int dtype, const void* Hpk, const void* W, const int32_t* tok,
+                      const float* lse, const float* coef, float* dH, float* dW, int flags, void* ws,
+                      size_t ws_bytes, ps_stream_t stream) {
+  NvtxRange nvtx_range("ps_lmhead_ppo_bwd");
+  return lmhead_bwd_impl(N, d, V, 0, dtype, Hpk, W, tok, lse, coef, dH, dW, flags, ws, ws_bytes, stream);
+}
+
+int ps_lmhead_ppo_bwd_vocab_shard(int64_t N, int d, int Vs, int64_t v0, int V, int dtype, const void* Hpk,
+                                  const void* W_shard, const int32_t* tok, const float* lse, const float* coef,
+                                  float* dH, float* dW_shard, int flags, void* ws, size_t ws_bytes,
+                                  ps_stream_t stream) {
+  NvtxRange nvtx_range("ps_lmhead_ppo_bwd_vocab_shard");
+  if (Vs < 1 || v0 < 0 || V < 1 || v0 + Vs > V) return PS_ERR_INVALID_ARG;
+  return lmhead_bwd_impl(N, d, Vs, v0, dtype, Hpk, W_shard, tok, lse, coef, dH, dW_shard, flags, ws, ws_bytes,
+                         stream);
 }
 
 // ----------------------------------------------------------------------------- diagnostics

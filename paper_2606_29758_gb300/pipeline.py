@@ -186,6 +186,81 @@ class DataParallelUpdate:
         return n
 
 
+def vocab_shards(V: int, S: int):
+    """S contiguous vocabulary ranges (v0, Vs) of sizes as equal as possible."""
+    if not 1 <= S <= V:
+        raise ValueError("need 1 <= S <= V")
+    return [(r * V // S, (r + 1) * V // S - r * V // S) for r in range(S)]
+
+
+class VocabParallelHead:
+    """The update pass's head split by vocabulary rows (the vocabulary-parallel calls of psppo.h).
+
+    `shards` lists the ranges (v0, Vs) of all S shards, in order; W_shard r is rows [v0, v0 + Vs)
+    of W. Per step: `stats(r, ...)` for every local shard, `gather()` (all_gather of the S shards'
+    12 bytes per row over `group`; nothing with one process, which then holds every shard), the
+    identical `forward(...)` on every process, `backward(r, ...)` for every local shard (its dW rows and
+    its term of dH, added into dH by every local shard after the first: PS_DH_ACCUMULATE), and
+    `reduce_dH()` (the all_reduce of dH over the processes; nothing with one process)."""
+
+    def __init__(self, shards, capacity: int, d: int, V: int, dtype: torch.dtype = torch.bfloat16,
+                 device: str = "cuda", eps: float = 0.2, loss_scale: float = 1.0, bwd_chunk_rows: int = 32768,
+                 group=None):
+        self.shards, self.d, self.V, self.eps, self.loss_scale, self.group = list(shards), d, V, eps, loss_scale, group
+        self.S = len(self.shards)
+        self.dcode = B.dtype_code(torch.empty(0, dtype=dtype))
+        f32 = dict(dtype=torch.float32, device=device)
+        u8 = dict(dtype=torch.uint8, device=device)
+        self.stats_all = torch.empty(self.S, capacity, 2, **f32)
+        self.ztok_all = torch.empty(self.S, capacity, **f32)
+        vmax = max(Vs for _, Vs in self.shards)
+        self.ws_stats = torch.zeros(B.ps_lmhead_logit_stats_workspace_size(capacity, d, vmax, self.dcode), **u8)
+        self.ws_fin = torch.zeros(B.ps_lmhead_ppo_fwd_from_stats_workspace_size(capacity), **u8)
+        self.capacity = capacity
+        self.chunk_rows = min(bwd_chunk_rows, capacity)
+        self.ws_bwd = torch.zeros(B.ps_lmhead_ppo_bwd_workspace_size(capacity, d, vmax, self.dcode, self.chunk_rows),
+                                  **u8)
+        self.lse, self.logp, self.ratio, self.coef, self.row_loss = (torch.empty(capacity, **f32) for _ in range(5))
+        self.loss = torch.zeros(1, dtype=torch.float64, device=device)
+
+    def stats(self, r: int, N: int, hid, W_shard, tok):
+        v0, Vs = self.shards[r]
+        B.ps_lmhead_logit_stats(N, self.d, Vs, v0, self.dcode, hid, W_shard, tok, self.stats_all[r], self.ztok_all[r],
+                                self.ws_stats)
+
+    def gather(self, N: int, rank: int):
+        """Every shard's statistics on every process (rank = the index of this process's shard)."""
+        import torch.distributed as dist
+        if not (dist.is_available() and dist.is_initialized()) or dist.get_world_size(self.group) == 1:
+            return
+        dist.all_gather([self.stats_all[r, :N] for r in range(self.S)], self.stats_all[rank, :N].clone(),
+                        group=self.group)
+        dist.all_gather([self.ztok_all[r, :N] for r in range(self.S)], self.ztok_all[rank, :N].clone(),
+                        group=self.group)
+
+    def forward(self, N: int, tok, oldlogp, adv, w):
+        ld = self.stats_all.shape[1]
+        B.ps_lmhead_ppo_fwd_from_stats(N, self.S, ld, self.V, self.stats_all, self.ztok_all, tok, oldlogp, adv, w,
+                                       self.eps, self.loss_scale,
+                                       self.loss, self.lse, self.logp, self.ratio, self.coef, self.row_loss,
+                                       self.ws_fin)
+
+    def backward(self, r: int, N: int, hid, W_shard, tok, dH, dW_shard, add_to_dH: bool = False):
+        """Shard r's rows of dW (overwritten) and its term of dH (written, or added to dH)."""
+        v0, Vs = self.shards[r]
+        # the workspace of chunk_rows rows at this shard's width: every shard (and the whole head with
+        # the same chunk_rows) cuts the rows into the same chunks
+        nb = B.ps_lmhead_ppo_bwd_workspace_size(self.capacity, self.d, Vs, self.dcode, self.chunk_rows)
+        B.ps_lmhead_ppo_bwd_vocab_shard(N, self.d, Vs, v0, self.V, self.dcode, hid, W_shard, tok, self.lse,
+                                        self.coef, dH, dW_shard, B.PS_DH_ACCUMULATE if add_to_dH else 0,
+                                        self.ws_bwd[:nb])
+
+    def reduce_dH(self, dH):
+        import torch.distributed as dist
+        if dist.is_available() and dist.is_initialized() and dist.get_world_size(self.group) > 1:
+            dist.all_reduce(dH, group=self.group)
+
+
 class InputStager:
     """Double-buffered host -> device staging of the unpacked batch inputs.
 

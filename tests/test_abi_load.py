@@ -99,3 +99,30 @@ def test_size_limits_and_design_arguments_are_rejected_on_the_host(lib):
     assert L.ps_design_cutoffs(1, 8, 10, fake, None, None, 4.0, 9, 0.0, fake, None, None, 0, None) == INV
     assert L.ps_design_cutoffs(1, 8, 10, fake, None, None, 4.0, 4, 0.5, fake, None, None, 0, None) == INV
     assert L.ps_design_cutoffs(1, 8, 10, fake, None, None, 0.0, 3, 0.0, fake, None, None, 0, None) == INV
+
+
+def test_vocabulary_shard_arguments_are_rejected_on_the_host(lib):
+    # The vocabulary-parallel calls check their shard and sizes before any CUDA call (no GPU here).
+    L = lib
+    INV = 1
+    stats = lambda N, d, Vs, v0, dt: L.ps_lmhead_logit_stats(N, d, Vs, v0, dt, None, None, None, None, None,  # noqa: E731
+                                                             None, 0, None)
+    assert stats(10, 128, 0, 0, 0) == INV           # an empty shard
+    assert stats(10, 128, 64, -1, 0) == INV         # a shard before token id 0
+    assert stats(-1, 128, 64, 0, 0) == INV
+    assert stats(10, 100, 64, 0, 0) == INV          # bf16 hidden size not a multiple of 8
+    assert stats(10, 128, 64, 0, 0) == INV          # rows but NULL pointers
+    fin = lambda N, S, ld, V: L.ps_lmhead_ppo_fwd_from_stats(N, S, ld, V, None, None, None, None, None, None,  # noqa: E731
+                                                             0.2, 1.0, None, None, None, None, None, None, None, 0,
+                                                             None)
+    assert fin(10, 0, 10, 1024) == INV              # no shard
+    assert fin(10, 2, 10, 0) == INV
+    assert fin(10, 2, 9, 1024) == INV               # shard stride below the rows
+    assert fin(10, 2, 10, 1024) == INV              # NULL loss
+    bwd = lambda N, Vs, v0, V: L.ps_lmhead_ppo_bwd_vocab_shard(N, 128, Vs, v0, V, 0, None, None, None, None,  # noqa: E731
+                                                               None, None, None, 0, None, 0, None)
+    assert bwd(10, 64, 1000, 1024) == INV           # the shard runs past the vocabulary
+    assert bwd(10, 64, -5, 1024) == INV
+    assert bwd(10, 0, 0, 1024) == INV
+    assert L.ps_lmhead_logit_stats_workspace_size(10, 128, 64, 0) == L.ps_lmhead_ppo_fwd_workspace_size(10, 128, 64, 0)
+    assert L.ps_lmhead_ppo_fwd_from_stats_workspace_size(1000) >= 256 + 8 * 4
