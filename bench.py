@@ -485,26 +485,35 @@ def _oracle_head(cfg, b, W64, pk, rows):
 
 
 def _oracle_timing(cfg, b, W64, rows, step):
-    """One step of the oracle, timed in two parts: the whole batch's cutoffs, advantages and packing
-    indices (in full), and the head over a sample of `rows` packed rows. The head's work is linear in
-    the rows (each row's forward and dH; dW sums block by block of 128 rows, each block touching all
-    of V x d, so a sample of whole blocks costs per row what a whole step does), so a whole step's
-    time is the prefix time plus N times the head's per-row time."""
+    """One step of the oracle, timed in parts: the whole batch's cutoffs, advantages and packing
+    indices (in full), then the head on the first rows/2 and the first `rows` packed rows (whole
+    128-row blocks of the oracle's head). A head call costs a fixed part (its V x d float64 dW
+    accumulator, allocated and touched once per call) plus a part linear in the rows; the two sample
+    sizes separate them, so a whole step is prefix + fixed + N x per-row."""
     t0 = time.perf_counter()
     pk = _oracle_prefix(cfg, b, step)
     t1 = time.perf_counter()
-    done = _oracle_head(cfg, b, W64, pk, rows)
+    small = _oracle_head(cfg, b, W64, pk, rows // 2)
     t2 = time.perf_counter()
-    return {"N": pk["N"], "prefix_s": t1 - t0, "head_rows": done, "head_s": t2 - t1}
+    large = _oracle_head(cfg, b, W64, pk, rows)
+    t3 = time.perf_counter()
+    return {"N": pk["N"], "prefix_s": t1 - t0, "rows": (small, large), "head_s": (t2 - t1, t3 - t2)}
 
 
 def _oracle_summary(ts):
     N = float(np.mean([t["N"] for t in ts]))
     prefix_s = float(np.mean([t["prefix_s"] for t in ts]))
-    head_rate = sum(t["head_rows"] for t in ts) / sum(t["head_s"] for t in ts)
-    step_s = prefix_s + N / head_rate
-    return {"value": N / step_s, "unit": "tokens/s", "head_rows_per_s": head_rate, "prefix_s_per_step": prefix_s,
-            "extrapolated_step_s": step_s, "mean_prefix_rows": N}
+    d_rows = sum(t["rows"][1] - t["rows"][0] for t in ts)
+    d_s = sum(t["head_s"][1] - t["head_s"][0] for t in ts)
+    if d_rows > 0 and d_s > 0:
+        per_row = d_s / d_rows
+        fixed = max(0.0, float(np.mean([t["head_s"][1] - t["rows"][1] * per_row for t in ts])))
+    else:   # samples too small to separate the two parts (timing noise): all of it per row
+        per_row = sum(t["head_s"][1] for t in ts) / max(1, sum(t["rows"][1] for t in ts))
+        fixed = 0.0
+    step_s = prefix_s + fixed + N * per_row
+    return {"value": N / step_s, "unit": "tokens/s", "head_rows_per_s": 1.0 / per_row, "head_fixed_s": fixed,
+            "prefix_s_per_step": prefix_s, "extrapolated_step_s": step_s, "mean_prefix_rows": N}
 
 
 def cpu_baseline(cfg, b, rows):
@@ -514,9 +523,10 @@ def cpu_baseline(cfg, b, rows):
     out = _oracle_summary([t])
     out.update({"cores": os.cpu_count(), "kind": "oracle",
                 "sample": f"one {cfg.name} step: cutoffs, advantages and packing indices of the whole batch "
-                          f"({t['prefix_s']:.2f} s), then the f64 head forward + dH + dW over {t['head_rows']} "
-                          f"packed rows ({t['head_s']:.1f} s); value = the step's packed rows / (prefix time + "
-                          f"rows x per-row head time), extrapolated"})
+                          f"({t['prefix_s']:.2f} s), then the f64 head forward + dH + dW over {t['rows'][0]} and "
+                          f"{t['rows'][1]} packed rows ({t['head_s'][0]:.1f} + {t['head_s'][1]:.1f} s): a fixed "
+                          f"{out['head_fixed_s']:.2f} s per head call plus {1e3 / out['head_rows_per_s']:.1f} ms per "
+                          f"row; value = the step's packed rows / (prefix + fixed + rows x per-row), extrapolated"})
     return out
 
 
@@ -550,11 +560,13 @@ def run_reference(args):
         "vs_baseline": None, "dtype": "f64", "data": "synthetic (seeded generator; random-init head)",
         "config": {"workload": describe(cfg), "sample_rows_per_step": args.ref_rows},
         "cpu_baseline": {"value": v, "unit": "tokens/s", "cores": os.cpu_count(), "kind": "oracle",
-                         "head_rows_per_s": summ["head_rows_per_s"], "prefix_s_per_step": summ["prefix_s_per_step"],
+                         "head_rows_per_s": summ["head_rows_per_s"], "head_fixed_s": summ["head_fixed_s"],
+                         "prefix_s_per_step": summ["prefix_s_per_step"],
                          "sample": f"{args.steps} steps, each: cutoffs, advantages and packing indices of the "
                                    f"whole batch in full, then the f64 head forward + dH + dW over "
-                                   f"{args.ref_rows} packed rows ({dt:.1f} s in all); value and ms_per_step = "
-                                   f"one whole step extrapolated: prefix time + N x per-row head time"},
+                                   f"{args.ref_rows // 2} and {args.ref_rows} packed rows ({dt:.1f} s in all); "
+                                   f"value and ms_per_step = one whole step extrapolated: prefix time + the head's "
+                                   f"fixed cost per call + N x its per-row cost"},
         "e2e": {"value": v, "unit": "tokens/s", "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
     }))
 
@@ -626,9 +638,9 @@ def main():
     ap.add_argument("--config", default=WORKLOAD)
     ap.add_argument("--chunk-rows", type=int, default=65536)
     ap.add_argument("--cpu-rows", type=int, default=256)
-    # whole 128-row blocks of the oracle's head (its dW update touches all of V x d once per block),
-    # so that the per-row cost of the sample is the per-row cost of a whole step
-    ap.add_argument("--ref-rows", type=int, default=128)
+    # the head is timed on ref_rows/2 and ref_rows packed rows, whole 128-row blocks of the oracle's
+    # head (its dW update touches all of V x d once per block), separating its per-call and per-row cost
+    ap.add_argument("--ref-rows", type=int, default=256)
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--no-design", action="store_true", help="skip timing the cutoff-design stage")
     ap.add_argument("--replicas", action="store_true",

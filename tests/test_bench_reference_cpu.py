@@ -10,7 +10,7 @@ ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
 
 def test_reference_arm_prints_one_contract_line():
     out = subprocess.run([sys.executable, os.path.join(ROOT, "bench.py"), "--impl", "reference", "--config", "tiny",
-                          "--steps", "1", "--warmup", "0", "--ref-rows", "8"],
+                          "--steps", "1", "--warmup", "0", "--ref-rows", "16"],
                          capture_output=True, text=True, timeout=600, cwd=ROOT,
                          env=dict(os.environ, CUDA_VISIBLE_DEVICES=""))
     assert out.returncode == 0, out.stderr[-2000:]
