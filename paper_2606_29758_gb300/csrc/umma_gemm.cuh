@@ -27,9 +27,7 @@ namespace psk {
 constexpr int kBM = 128;
 constexpr int kBN = 256;
 constexpr int kBK = 64;
-constexpr int kStages = 4;
 constexpr int kGemmThreads = 192;
-constexpr int kEpiWarp0 = 2;
 constexpr uint32_t kTileABytes = kBM * kBK * 2;   // 16 KB
 constexpr uint32_t kTileBBytes = kBN * kBK * 2;   // 32 KB
 constexpr uint32_t kTmemCols = 512;               // two 256-column f32 accumulators
@@ -91,7 +89,6 @@ struct GemmSmemT {
 };
 template <int HALVES>
 constexpr size_t gemm_smem_bytes() { return sizeof(GemmSmemT<HALVES>) + 1024; }  // + alignment slack
-constexpr size_t kGemmSmemBytes = gemm_smem_bytes<1>();
 
 // tmC: the output map of epilogues that store through TMA (unused by the others).
 template <bool A_MN, bool B_MN, class Epi, int HALVES = 1>
