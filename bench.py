@@ -40,9 +40,9 @@ MEASURED_PEAKS = os.path.join(ROOT, "MEASURED_PEAKS.json")
 FALLBACK_PEAKS = {"hbm_gbs": 6800.0, "bf16_tflops": 1900.0, "bf16_tflops_sustained": 1700.0}
 
 # DRAM bytes (read + write) per launch of the forward GEMM on the 7b workload, the mean of the
-# six launches in profiles/lmhead_pass_7b_launch_list.md (53.15 GB read + 0.92 GB written).
+# six launches in profiles/lmhead_pass_7b_launch_list.md (55.39 GB read + 0.92 GB written).
 # Reset to None whenever the forward kernel or its schedule changes.
-FWD_GEMM_TRAFFIC = {"7b": 54.07e9}
+FWD_GEMM_TRAFFIC = {"7b": 56.31e9}
 
 
 def describe(cfg) -> str:
@@ -322,6 +322,42 @@ def run_ours(args):
             return {"error": f"{type(e).__name__}: {e}"}
 
     full_control = optional(full_control_run)
+
+    # ---- context: the same step with the head split into vocabulary shards (VocabParallelHead), the
+    # shards run one after another on this device: what the split itself costs
+    def vocab_parallel_run(S):
+        from paper_2606_29758_gb300 import VocabParallelHead, vocab_shards
+        shards = vocab_shards(cfg.V, S)
+        vp = VocabParallelHead(shards, b.total_len, cfg.d, cfg.V, tdtype, device=dev, eps=cfg.eps,
+                               loss_scale=up.loss_scale, bwd_chunk_rows=args.chunk_rows)
+        W = D["W"]
+
+        def vstep(i):
+            up.sample(D["q"], D["L"], seed, i, traj_base=dpu.traj_base)
+            n = up.pack(D["L"], D["R"], D["tok_full"], D["oldlogp_full"], D["hid_full"])
+            for r, (v0, Vs) in enumerate(shards):
+                vp.stats(r, n, up.hid, W[v0:v0 + Vs], up.tok)
+            vp.forward(n, up.tok, up.oldlogp, up.adv, up.w)
+            for r, (v0, Vs) in enumerate(shards):
+                vp.backward(r, n, up.hid, W[v0:v0 + Vs], up.tok, up.dH, up.dW[v0:v0 + Vs], add_to_dH=r > 0)
+            return n
+
+        for i in range(2):
+            vstep(4000 + i)
+        barrier()
+        v0e, v1e = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        v0e.record(stream)
+        v_rows = sum(vstep(i) for i in range(3))
+        v1e.record(stream)
+        barrier()
+        v_ms = v0e.elapsed_time(v1e) / 3
+        del vp
+        return {"shards": S, "ms_per_step": v_ms, "tokens_per_s": v_rows / (v_ms * 3e-3),
+                "step_time_ratio_over_whole_head": v_ms / (ms / args.steps),
+                "note": "the same steps with W split into vocabulary shards run one after another on this device "
+                        "(logit statistics per shard, the forward from them, each shard's backward); 3 timed steps"}
+
+    vocab_parallel = optional(vocab_parallel_run, args.vocab_shards) if args.vocab_shards > 0 else None
     if args.no_design:
         design = None
     elif cfg.dtype != "bf16":
@@ -415,6 +451,7 @@ def run_ours(args):
                 "h2d_alone_ms": h2d_ms, "h2d_alone_gbs": h2d / (h2d_ms * 1e-3) / 1e9,
                 "overlap": "next batch copied on a second stream during the current pass (InputStager)"},
         "full_control": full_control,
+        **({"vocab_parallel": vocab_parallel} if vocab_parallel is not None else {}),
         "gpu_launches": launches,
         "clocks": clk,
     }
@@ -643,6 +680,8 @@ def main():
     ap.add_argument("--ref-rows", type=int, default=256)
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--no-design", action="store_true", help="skip timing the cutoff-design stage")
+    ap.add_argument("--vocab-shards", type=int, default=0,
+                    help="also time the step with the head split into this many vocabulary shards (context)")
     ap.add_argument("--replicas", action="store_true",
                     help="with several ranks: independent replicas, no exchange of dW")
     args = ap.parse_args()
