@@ -10,12 +10,17 @@ The batch is the f32 Tiny workload (so dZ is not rounded to bf16) with a cutoff 
 half its mass at T_p: every xi_t >= 1/2, the weights stay <= 2 and the Monte Carlo mean is close
 to Gaussian. The same comparison against the mean a pass without the 1/xi weights would have
 (a mistake planted in the oracle's reference) must fail by a wide margin.
+
+The zero-cutoff mode runs the same check with masses that cover 3/4 of 2^62: the deficit is
+Pr(H = 0) = 1/4 (a draw keeps no token of its completion, as an optimised design of Appendix F
+allows), xi_t = Pr(H >= t) counts it (xi_1 = 3/4) and the weights are 1/xi_t of that distribution;
+a reference whose weights ignore the deficit (xi_1 = 1) must fail as well.
 """
 import numpy as np
 import pytest
 
 from oracle import lmhead
-from oracle.cutoffs import ONE62, xi
+from oracle.cutoffs import ONE62, survival_with_zero, xi
 from oracle.pack import group_advantages, pack_prefixes
 from synthetic import get_config, make_batch
 
@@ -24,7 +29,7 @@ pytestmark = pytest.mark.gpu
 M = 512
 
 
-def _half_at_end_masses(L, K, T_max):
+def _half_at_end_masses(L, K, T_max, zero=False):
     P = len(L) // K
     q = np.zeros((P, T_max), dtype=np.uint64)
     for p in range(P):
@@ -32,12 +37,19 @@ def _half_at_end_masses(L, K, T_max):
         each = (1 << 61) // T
         q[p, :T] = each
         q[p, T - 1] += ONE62 - each * T
+    if zero:
+        q = (q // 4) * 3                        # Pr(H = 0) = 1/4 (up to 2^-62 per mass)
     return q
 
 
-def _oracle_full_and_variance(cfg, b, q):
-    """Full-trajectory dW and hidden-state gradient, and the per-coordinate variance of one draw
-    of the truncated estimator."""
+def _survival(q_p, zero):
+    return np.array([v / ONE62 for v in survival_with_zero(q_p)]) if zero else xi(q_p)
+
+
+def _oracle_full_and_variance(cfg, b, q, zero=False):
+    """Full-trajectory dW and hidden-state gradient, the per-coordinate variance of one draw of the
+    truncated estimator, and the means of two mistaken passes: one without the 1/xi weights, one
+    whose weights take the masses as covering 2^62."""
     K = cfg.K
     L = b.L.astype(np.int64)
     A = group_advantages(b.R, K, cfg.adv_mode)
@@ -50,7 +62,7 @@ def _oracle_full_and_variance(cfg, b, q):
     var_w = np.zeros_like(dW)
     var_h = np.zeros_like(dH)
     for k in range(len(L)):
-        x = xi(q[k // K])[:L[k]]               # t <= L_k <= T_p, so xi_t >= 1/2 here
+        x = _survival(q[k // K], zero)[:L[k]]  # t <= L_k <= T_p, so xi_t >= 1/2 (3/8 with a deficit)
         c = 1.0 / x - 1.0
         rows = np.nonzero(pk["row_traj"] == k)[0]
         rows = rows[np.argsort(pk["row_pos"][rows])]
@@ -66,21 +78,26 @@ def _oracle_full_and_variance(cfg, b, q):
     dhid = np.zeros((len(b.tok_full), cfg.d))
     dhid[pk["src_row"]] = dH
     # what the mean would be without the 1/xi weights: each token kept with probability xi_t
-    keep = np.array([xi(q[int(pk["row_traj"][i]) // K])[int(pk["row_pos"][i]) - 1] for i in range(len(pk["tok"]))])
+    idx = (pk["row_traj"] // K, pk["row_pos"] - 1)
+    keep = np.stack([_survival(q_p, zero) for q_p in q])[idx]
     dW_unweighted = (keep[:, None] * dz).T @ H
-    return dW, dhid, var_w, var_h, dW_unweighted
+    # weights 1/xi'_t with xi'_t = 1 - U[t-1]/2^62 (the deficit ignored): the mean is xi_t / xi'_t dz
+    dW_wrong_xi = ((keep / np.stack([xi(q_p) for q_p in q])[idx])[:, None] * dz).T @ H
+    return dW, dhid, var_w, var_h, dW_unweighted, dW_wrong_xi
 
 
-def test_monte_carlo_mean_of_the_cuda_pass_is_the_full_gradient():
+@pytest.mark.parametrize("zero", [False, True], ids=["trunc", "trunc_zero"])
+def test_monte_carlo_mean_of_the_cuda_pass_is_the_full_gradient(zero):
     import torch
-    from paper_2606_29758_gb300 import PassShape, UpdatePass
+    from paper_2606_29758_gb300 import PS_MODE_TRUNC, PS_MODE_TRUNC_ZERO, PassShape, UpdatePass
     cfg = get_config("tiny")
     b = make_batch(cfg, device="cuda")
-    q = _half_at_end_masses(b.L, cfg.K, b.T_max)
+    q = _half_at_end_masses(b.L, cfg.K, b.T_max, zero)
     D = dict(b.dev)
     D["q"] = torch.from_numpy(q.view(np.int64)).cuda()
     up = UpdatePass(PassShape(cfg.P, cfg.K, b.T_max, cfg.d, cfg.V, b.total_len, torch.float32),
-                    eps=cfg.eps, loss_scale=cfg.loss_scale, adv_mode=cfg.adv_mode)
+                    eps=cfg.eps, loss_scale=cfg.loss_scale, adv_mode=cfg.adv_mode,
+                    mode=PS_MODE_TRUNC_ZERO if zero else PS_MODE_TRUNC)
     acc_w = torch.zeros(cfg.V, cfg.d, dtype=torch.float64, device="cuda")
     acc_h = torch.zeros(b.total_len, cfg.d, dtype=torch.float64, device="cuda")
     kept = 0
@@ -94,7 +111,7 @@ def test_monte_carlo_mean_of_the_cuda_pass_is_the_full_gradient():
     mean_w = acc_w.cpu().numpy() / M
     mean_h = acc_h.cpu().numpy() / M
 
-    dW, dhid, var_w, var_h, dW_unweighted = _oracle_full_and_variance(cfg, b, q)
+    dW, dhid, var_w, var_h, dW_unweighted, dW_wrong_xi = _oracle_full_and_variance(cfg, b, q, zero)
     assert kept < M * b.total_len          # the passes really truncated
     floor_w = (1e-6 * np.abs(dW).max()) ** 2
     floor_h = (1e-6 * np.abs(dhid).max()) ** 2
@@ -106,3 +123,6 @@ def test_monte_carlo_mean_of_the_cuda_pass_is_the_full_gradient():
     # the planted mistake: a reference without the inverse-survival weights is rejected
     z_bad = (mean_w - dW_unweighted) / np.sqrt(var_w / M + floor_w)
     assert np.abs(z_bad).max() > 12.0, np.abs(z_bad).max()
+    if zero:
+        z_bad = (mean_w - dW_wrong_xi) / np.sqrt(var_w / M + floor_w)
+        assert np.abs(z_bad).max() > 12.0, np.abs(z_bad).max()

@@ -7,7 +7,7 @@ import numpy as np
 import pytest
 
 from oracle import lmhead
-from oracle.cutoffs import ONE62, inverse_survival_weights, sample_cutoffs, xi
+from oracle.cutoffs import ONE62, cumulative_masses, inverse_survival_weights, sample_cutoffs, xi
 from oracle.pack import group_advantages, pack_prefixes
 from synthetic.generate import beta_masses
 
@@ -27,11 +27,15 @@ def _setup(seed=0, L=(6, 9), d=4, V=13):
     return dict(L=L, K=K, q=q, hid=hid, W=W, tok=tok, old=old, R=R, c=1.0 / K, eps=0.2)
 
 
-def _grads_for_cutoffs(s, H, mode="trunc"):
-    """Gradients w.r.t. W and w.r.t. the unpacked hidden states for given cutoffs."""
+def _grads_for_cutoffs(s, H, mode="trunc", w_tab=None):
+    """Gradients w.r.t. W and w.r.t. the unpacked hidden states for given cutoffs (H = 0 keeps no
+    token of its completion); w_tab overrides the weights 1/xi_t of the masses."""
     L = s["L"]
     n = np.minimum(H, L) if mode == "trunc" else L.astype(np.int64)
-    w_tab = inverse_survival_weights(s["q"][0])[None] if mode == "trunc" else np.ones_like(s["q"], dtype=np.float64)
+    if w_tab is None:
+        w_tab = inverse_survival_weights(s["q"][0])[None] if mode == "trunc" else np.ones_like(s["q"], dtype=np.float64)
+    if n.sum() == 0:
+        return np.zeros_like(s["W"]), np.zeros_like(s["hid"])
     A = group_advantages(s["R"], s["K"], 1)
     pk = pack_prefixes(L, n, s["K"], w_tab, A, s["tok"], s["old"], s["hid"])
     f = lmhead.forward(pk["hid"], s["W"], pk["tok"], pk["oldlogp"], pk["adv"], pk["w"], s["eps"], s["c"])
@@ -107,3 +111,39 @@ def test_monte_carlo_mean_within_exact_sampling_error():
     zscore = (mean - GW) / np.sqrt(var / M + 1e-300)
     assert np.abs(zscore).max() < 4.5
     assert np.abs(mean - GW).max() > 0  # the estimate is random, not the full update itself
+
+
+def _deficit_setup():
+    # masses summing to 3/4 of 2^62: the deficit, Pr(H = 0) = 1/4, keeps no token of a completion
+    # (the zero-cutoff sampling of an optimised design, Appendix F, where xi_1 < 1)
+    s = _setup(seed=5, L=(5, 8))
+    s["q"] = (s["q"] // 4) * 3
+    return s
+
+
+def _enumerate_with_zero(s, w_tab):
+    T = int(s["L"].max())
+    U = cumulative_masses(s["q"][0])
+    p = [(ONE62 - U[-1]) / ONE62] + [int(m) / ONE62 for m in s["q"][0]]      # h = 0, 1, ..., T
+    EW, Ehid = 0.0, 0.0
+    for hs in itertools.product(range(T + 1), repeat=s["K"]):
+        pr = float(np.prod([p[h] for h in hs]))
+        dW, dhid = _grads_for_cutoffs(s, np.array(hs), w_tab=w_tab)
+        EW = EW + pr * dW
+        Ehid = Ehid + pr * dhid
+    return EW, Ehid
+
+
+def test_exact_enumeration_with_zero_cutoffs_equals_full_update():
+    s = _deficit_setup()
+    assert 0.24 < (ONE62 - cumulative_masses(s["q"][0])[-1]) / ONE62 < 0.26
+    w = inverse_survival_weights(s["q"][0], allow_zero=True)
+    assert w[0] == pytest.approx(ONE62 / float(cumulative_masses(s["q"][0])[-1]), rel=1e-15)   # 1/xi_1 = 4/3
+    EW, Ehid = _enumerate_with_zero(s, w[None])
+    GW, Ghid = _grads_for_cutoffs(s, None, mode="full")
+    np.testing.assert_allclose(EW, GW, rtol=1e-11, atol=1e-13 * np.abs(GW).max())
+    np.testing.assert_allclose(Ehid, Ghid, rtol=1e-11, atol=1e-13 * np.abs(Ghid).max())
+    # planted mistake: weights taken as if the masses covered 2^62 (xi_1 = 1) leave the mean biased
+    w_bad = np.array([ONE62 / float(ONE62 - u) for u in cumulative_masses(s["q"][0])[:-1]])
+    EW_bad, _ = _enumerate_with_zero(s, w_bad[None])
+    assert np.abs(EW_bad - GW).max() > 0.1 * np.abs(GW).max()
