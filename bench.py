@@ -8,7 +8,11 @@ cutoffs (the Philox step counter advances), so N varies from step to step.
 
 value: prefix tokens/s, whole job (sum of packed rows over all steps and ranks divided
 by the max over ranks of the device-timed region). The credited work of a step is
-6 N d V FLOPs (forward GEMM, dH, dW; the backward's logit recompute is not credited).
+6 N d V FLOPs (forward GEMM, dH, dW). By default the forward keeps its logits in the
+logit store where the device memory holds it (about 60 GB at the 7B workload), and the
+backward turns them into dZ in place instead of recomputing them (executing 6 N d V
+rather than 8 N d V); --logits recompute times the recomputing backward, and the line's
+recompute_control does so on the same batch in every run.
 
     python bench.py [--gpus N] [--steps K] [--warmup W] [--impl ours|reference|torch]
 
@@ -42,7 +46,7 @@ FALLBACK_PEAKS = {"hbm_gbs": 6800.0, "bf16_tflops": 1900.0, "bf16_tflops_sustain
 # DRAM bytes (read + write) per launch of the forward GEMM on the 7b workload, the mean of the
 # six launches in profiles/lmhead_pass_7b_launch_list.md (55.39 GB read + 0.92 GB written).
 # Reset to None whenever the forward kernel or its schedule changes.
-FWD_GEMM_TRAFFIC = {"7b": 56.31e9}
+FWD_GEMM_TRAFFIC = {("7b", "FwdLseEpi"): 56.31e9}
 
 
 def describe(cfg) -> str:
@@ -122,6 +126,21 @@ def _dist():
     return world, rank, local
 
 
+def logit_store_rows(args, cfg, b, dev):
+    """Rows of the logit store: 0 (recompute the logits in the backward), or as many of the batch's
+    sum of lengths (the largest N a step can have) as fit in the device memory left after the pass's
+    other buffers, with a margin."""
+    import torch
+
+    from paper_2606_29758_gb300 import ps_lmhead_logit_store_size
+    if args.logits == "recompute" or cfg.dtype != "bf16":
+        return 0
+    free, _ = torch.cuda.mem_get_info(dev)
+    other = 40e9 + b.total_len * cfg.d * 12.0 + cfg.V * cfg.d * 8.0 + args.chunk_rows * cfg.V * 2.0
+    per_row = ps_lmhead_logit_store_size(1 << 16, cfg.V) / (1 << 16)
+    return int(max(0, min(b.total_len, (free - other) // per_row)))
+
+
 def run_ours(args):
     import torch
     import torch.distributed as dist
@@ -138,7 +157,8 @@ def run_ours(args):
     b = make_batch(cfg, device=dev)
     D = b.dev
     tdtype = torch.bfloat16 if cfg.dtype == "bf16" else torch.float32
-    shape = PassShape(cfg.P, cfg.K, b.T_max, cfg.d, cfg.V, b.total_len, tdtype, args.chunk_rows)
+    store_rows = logit_store_rows(args, cfg, b, dev)
+    shape = PassShape(cfg.P, cfg.K, b.T_max, cfg.d, cfg.V, b.total_len, tdtype, args.chunk_rows, store_rows)
     # data-parallel: every rank's completions are a slice of one global batch of world x P prompts
     dp = world > 1 and not args.replicas
     up = UpdatePass(shape, device=dev, eps=cfg.eps, loss_scale=cfg.loss_scale / world if dp else cfg.loss_scale)
@@ -323,6 +343,31 @@ def run_ours(args):
 
     full_control = optional(full_control_run)
 
+    # ---- control: the same steps with the logits recomputed in the backward instead of kept
+    def recompute_control_run():
+        up.use_store = False
+        try:
+            for i in range(2):
+                step(3500 + i)
+            barrier()
+            r0 = torch.cuda.Event(enable_timing=True)
+            r1 = torch.cuda.Event(enable_timing=True)
+            r_steps = 3
+            r0.record(stream)
+            r_rows = sum(step(3600 + i) for i in range(r_steps))
+            r1.record(stream)
+            barrier()
+        finally:
+            up.use_store = True
+        up.check_status()
+        r_ms = r0.elapsed_time(r1) / r_steps
+        return {"ms_per_step": r_ms, "tokens_per_s": r_rows / (r_ms * r_steps * 1e-3),
+                "step_time_ratio_over_store": r_ms / (ms / args.steps),
+                "note": "the same prefix steps with the logits recomputed by the backward (chunks of "
+                        f"{args.chunk_rows} rows) instead of kept in the logit store; 3 timed steps"}
+
+    recompute_control = optional(recompute_control_run) if store_rows > 0 else None
+
     # ---- context: the same step with the head split into vocabulary shards (VocabParallelHead), the
     # shards run one after another on this device: what the split itself costs
     def vocab_parallel_run(S):
@@ -368,6 +413,9 @@ def run_ours(args):
     peaks, src = _peaks()
     d, V = cfg.d, cfg.V
     mean_rows = rows / args.steps
+    stored = [n <= store_rows for n in step_rows]      # steps whose forward kept the logits
+    all_stored = all(stored)
+    executed = 6.0 if all_stored else 8.0               # executed FLOPs per row, in units of d V
     t_fwd = float(per[:, 2].mean()) * 1e-3
     fwd_flops = 2.0 * mean_rows * d * V
     peak_tf = peaks["bf16_tflops_sustained"]
@@ -382,9 +430,10 @@ def run_ours(args):
     mhz_run = clk.get("sm_mhz") or None
     mhz_max = clk.get("sm_max_mhz") or peaks.get("sm_max_mhz", 2070.0)
     if cfg.dtype == "bf16":
-        roofline = {"kernel": "umma_gemm_kernel<K,K,FwdLseEpi> (fused forward; + O(N) finalize)",
+        fwd_kernel = "FwdLseStoreEpi" if all_stored else "FwdLseEpi"
+        roofline = {"kernel": f"umma_gemm_kernel<K,K,{fwd_kernel}> (fused forward; + O(N) finalize)",
                     "bound": "tensor", "achieved": achieved_tf, "peak": peak_tf, "unit": "TFLOP/s",
-                    "frac": achieved_tf / peak_tf, "traffic": FWD_GEMM_TRAFFIC.get(cfg.name),
+                    "frac": achieved_tf / peak_tf, "traffic": FWD_GEMM_TRAFFIC.get((cfg.name, fwd_kernel)),
                     "algorithmic_per_launch": f"2*N*d*V = {fwd_flops:.4g} FLOP",
                     "peak_note": f"bf16_tflops_sustained ({src}); kernel timed inside the step"}
     else:
@@ -395,8 +444,9 @@ def run_ours(args):
                     "traffic": None, "algorithmic_per_launch": f"2*N*d*V = {fwd_flops:.4g} FLOP",
                     "peak_note": "FP32 FMA lanes x 2 x maximum SM clock (derived, not measured)"}
     # per step: sampler 1, packing 2, forward 3 (GEMM, finalize, loss reduction), backward 3 per
-    # chunk (recompute, dH, dW); the backward splits a step's rows into ceil(N / chunk) chunks
-    launches = sum(6 + 3 * (-(-n // args.chunk_rows)) for n in step_rows)
+    # chunk (recompute, dH, dW; the backward splits a step's rows into ceil(N / chunk) chunks), or,
+    # from the logit store, 3 (conversion to dZ, dH, dW over all rows)
+    launches = sum(6 + (3 if st else 3 * (-(-n // args.chunk_rows))) for n, st in zip(step_rows, stored))
     out = {
         "metric": "prefix tokens/s (fused LM-head PS-PPO fwd+bwd, 1xGB300)",
         "value": rows_all / (ms_max * 1e-3),
@@ -413,8 +463,14 @@ def run_ours(args):
         "config": {"workload": describe(cfg),
                    "global_batch": cfg.B * world, "mean_prefix_rows": mean_rows, "sum_lengths": b.total_len,
                    "bwd_chunk_rows": args.chunk_rows,
+                   "logits": (f"kept by the forward in the logit store ({store_rows} rows, "
+                              f"{up.store.numel() / 1e9:.1f} GB), turned into dZ in place by the backward"
+                              if all_stored else "recomputed by the backward" if not any(stored)
+                              else f"store for steps of up to {store_rows} rows, recomputed above"),
                    "l2": f"inputs larger than L2 (hidden states {b.total_len * cfg.d * 2 / 1e9:.1f} GB, "
-                         f"W {cfg.V * cfg.d * 2 / 1e9:.2f} GB, dZ chunk {args.chunk_rows * cfg.V * 2 / 1e9:.1f} GB)",
+                         f"W {cfg.V * cfg.d * 2 / 1e9:.2f} GB, "
+                         + (f"logit store {mean_rows * cfg.V * 2 / 1e9:.1f} GB per step)" if all_stored else
+                            f"dZ chunk {args.chunk_rows * cfg.V * 2 / 1e9:.1f} GB)"),
                    "parallelism": ("data-parallel: prompt shards (global batch = ranks x P prompts, cutoffs "
                                    "by global completion index), dW and loss all-reduced over NCCL" if dp
                                    else "replicas" if world > 1 else "single GPU")},
@@ -427,8 +483,9 @@ def run_ours(args):
                           "arch_tflops_at_max_clock": arch_per_mhz * mhz_max,
                           "of_arch_at_max_clock": credited_tf / (arch_per_mhz * mhz_max),
                           "of_nominal_2250": credited_tf / 2250.0,
-                          "executed_8NdV_tflops": credited_tf * 8 / 6,
-                          "executed_of_arch_at_run_clock": (credited_tf * 8 / 6) / (arch_per_mhz * mhz_run)
+                          "executed_tflops": credited_tf * executed / 6,
+                          "executed_flops_per_row": f"{executed:.0f} d V",
+                          "executed_of_arch_at_run_clock": (credited_tf * executed / 6) / (arch_per_mhz * mhz_run)
                           if mhz_run else None,
                           "arch_note": f"{sms} SMs x 8192 dense bf16 FLOP per SM per clock x SM clock (run: median "
                                        f"sampled under load; max: the clock limit); nominal 2250 TFLOP/s dense; "
@@ -440,10 +497,13 @@ def run_ours(args):
                                 "all-reduce of dW and the loss (data-parallel runs only)"},
         "pass_stats": pass_stats,
         "roofline": roofline,
-        "roofline_backward": ({"kernels": "recompute + dH + dW GEMMs (executed 6*N*d*V per step)", "bound": "tensor",
-                               "achieved": 6.0 * mean_rows * d * V / (float(per[:, 3].mean()) * 1e-3) / 1e12,
+        "roofline_backward": ({"kernels": ("logit-store conversion + dH + dW GEMMs (executed 4*N*d*V per step)"
+                                           if all_stored else "recompute + dH + dW GEMMs (executed 6*N*d*V per step)"),
+                               "bound": "tensor",
+                               "achieved": (executed - 2) * mean_rows * d * V / (float(per[:, 3].mean()) * 1e-3) / 1e12,
                                "peak": peak_tf, "unit": "TFLOP/s",
-                               "frac": 6.0 * mean_rows * d * V / (float(per[:, 3].mean()) * 1e-3) / 1e12 / peak_tf,
+                               "frac": (executed - 2) * mean_rows * d * V / (float(per[:, 3].mean()) * 1e-3) / 1e12
+                               / peak_tf,
                                "traffic": None, "peak_note": "bf16_tflops_sustained"}
                               if cfg.dtype == "bf16" else None),
         "e2e": {"value": e_rows / (e_ms * 1e-3), "unit": "tokens/s", "h2d_bytes_per_step": h2d,
@@ -451,6 +511,7 @@ def run_ours(args):
                 "h2d_alone_ms": h2d_ms, "h2d_alone_gbs": h2d / (h2d_ms * 1e-3) / 1e9,
                 "overlap": "next batch copied on a second stream during the current pass (InputStager)"},
         "full_control": full_control,
+        **({"recompute_control": recompute_control} if recompute_control is not None else {}),
         **({"vocab_parallel": vocab_parallel} if vocab_parallel is not None else {}),
         "gpu_launches": launches,
         "clocks": clk,
@@ -674,6 +735,9 @@ def main():
     ap.add_argument("--torch-chunk", type=int, default=16384, help="rows per logit chunk of --impl torch")
     ap.add_argument("--config", default=WORKLOAD)
     ap.add_argument("--chunk-rows", type=int, default=65536)
+    ap.add_argument("--logits", choices=["recompute", "store"], default="store",
+                    help="keep the logits from the forward (logit store, where the device memory holds it) or "
+                         "recompute them in the backward")
     ap.add_argument("--cpu-rows", type=int, default=256)
     # the head is timed on ref_rows/2 and ref_rows packed rows, whole 128-row blocks of the oracle's
     # head (its dW update touches all of V x d once per block), separating its per-call and per-row cost

@@ -198,6 +198,48 @@ int ps_lmhead_ppo_bwd(int64_t N, int d, int V, int dtype, const void* Hpk, const
                       void* ws, size_t ws_bytes, ps_stream_t stream);
 
 /* ---------------------------------------------------------------------------
+ * Logit store: the forward keeps the head's logits for the backward, which then
+ * executes 4NdV instead of 6NdV FLOPs (no recomputation), at the price of N x V
+ * 2-byte values of device memory (about 60 GB for 2e5 rows of a 152k vocabulary).
+ * The same loss and gradients as ps_lmhead_ppo_fwd / ps_lmhead_ppo_bwd (Eq. 1,
+ * the head of Appendix D); bf16 only (PS_DTYPE_F32: PS_ERR_UNSUPPORTED).
+ *
+ * ps_lmhead_logit_store_size(N, V): bytes of the store of N rows (0 for bad args).
+ * Layout (owned by the caller, 16-byte aligned, written by the forward and
+ * consumed by the backward of the same N, Hpk, W and tok):
+ *   [N][ldz] 2-byte values, ldz = V rounded up to a multiple of 8: after the forward
+ *   f16 e_iv = 2^(x_iv - m_ic) with x = z log2(e), for the 32-column slice c = v / 32,
+ *   where m_ic is a running maximum of row i's x over the forward's sweep, at least
+ *   the largest x of slice c (so e is in [0, 1]; relative precision 2^-11 above 2^-14);
+ *   then, from byte offset ceil(N * ldz * 2 / 256) * 256, f32 m [ceil(V/32)][N].
+ * ps_lmhead_ppo_fwd_store: ps_lmhead_ppo_fwd (same arguments, outputs, workspace,
+ *   limits and errors) that also fills the store. store_bytes below
+ *   ps_lmhead_logit_store_size(N, V): PS_ERR_WORKSPACE, nothing launched.
+ * ps_lmhead_ppo_bwd_from_store: the backward of ps_lmhead_ppo_bwd from the store,
+ *   which it overwrites in place with dZ [N][ldz] bf16:
+ *     dZ_iv = coef_i (1[v = tok_i] - e_iv 2^(m_ic - lse_i log2(e))) for v != tok_i,
+ *     dZ_i,tok_i = coef_i (1 - exp(logp_i)) from the forward's logp,
+ *   then dH = dZ W and dW = dZ^T Hpk over all N rows (flags PS_DW_ACCUMULATE,
+ *   PS_DH_ACCUMULATE as for ps_lmhead_ppo_bwd; dH or dW may be NULL). lse, logp and
+ *   coef are the forward's outputs. Workspace: the status header,
+ *   ps_lmhead_ppo_bwd_from_store_workspace_size() bytes. Calling it twice on one
+ *   store is an error the library cannot see (the second call reads dZ as e).
+ * ------------------------------------------------------------------------- */
+size_t ps_lmhead_logit_store_size(int64_t N, int V);
+int ps_lmhead_ppo_fwd_store(int64_t N, int d, int V, int dtype, const void* Hpk, const void* W,
+                            const int32_t* tok, const float* oldlogp, const float* adv,
+                            const float* w, double eps, double loss_scale,
+                            double* loss, float* lse, float* logp, float* ratio, float* coef,
+                            float* row_loss, void* store, size_t store_bytes,
+                            void* ws, size_t ws_bytes, ps_stream_t stream);
+size_t ps_lmhead_ppo_bwd_from_store_workspace_size(void);
+int ps_lmhead_ppo_bwd_from_store(int64_t N, int d, int V, int dtype, const void* Hpk,
+                                 const void* W, const int32_t* tok, const float* lse,
+                                 const float* logp, const float* coef,
+                                 void* store, size_t store_bytes, float* dH, float* dW,
+                                 int flags, void* ws, size_t ws_bytes, ps_stream_t stream);
+
+/* ---------------------------------------------------------------------------
  * Vocabulary-parallel head: W split by vocabulary rows across devices.
  *
  * The same loss and gradients as ps_lmhead_ppo_fwd / ps_lmhead_ppo_bwd (Eq. 1 through

@@ -18,6 +18,11 @@ int fwd_tile_splits_bf16(int V);   // one partial per 256-column vocabulary tile
 int choose_fwd_splits_bf16(int64_t N, int d, int V, int num_sms, int max_splits);
 int fwd_gemm_bf16(int64_t N, int d, int V, const void* Hpk, const void* W, const int32_t* tok, float2* part,
                   float* ztok, int splits, uint32_t* status, cudaStream_t s, int tok_base = 0);
+// The same forward keeping its logits (the logit store): store [N][ldz] f16 with e = 2^(x - m) per
+// 32-column slice, m the running row maximum after the slice (log2 units), in scale [ceil(V/32)][N].
+int fwd_gemm_store_bf16(int64_t N, int d, int V, const void* Hpk, const void* W, const int32_t* tok, float2* part,
+                        float* ztok, int splits, void* store, int64_t ldz, float* scale, uint32_t* status,
+                        cudaStream_t s);
 int fwd_splits_f32(int V);
 int fwd_gemm_f32(int64_t N, int d, int V, const float* Hpk, const float* W, const int32_t* tok, float2* part,
                  float* ztok, uint32_t* status, cudaStream_t s, int tok_base = 0);
@@ -38,6 +43,12 @@ int proxy_topk_gemm_bf16(int64_t N, int d, int V, const void* Hrows, const void*
 int bwd_chunk_bf16(int64_t rc, int d, int V, const void* Hpk, const void* W, const int32_t* tok,
                    const float* lse, const float* coef, float* dH, float* dW, int dw_accumulate, void* dz,
                    int64_t ldz, uint32_t* status, cudaStream_t s, int tok_base = 0, int dh_accumulate = 0);
+// dH = dZ W and dW (+)= dZ^T Hpk from dZ [rc][ldz] bf16 already in memory.
+int bwd_grads_bf16(int64_t rc, int d, int V, const void* Hpk, const void* W, float* dH, float* dW, int dw_accumulate,
+                   const void* dz, int64_t ldz, uint32_t* status, cudaStream_t s, int dh_accumulate);
+// The logit store of the forward turned into dZ in place (f16 e -> bf16 dZ), rows [0, N).
+int dz_from_store_bf16(int64_t N, int V, void* store, int64_t ldz, const float* scale, const int32_t* tok,
+                       const float* lse, const float* logp, const float* coef, cudaStream_t s);
 int bwd_chunk_f32(int64_t rc, int d, int V, const float* Hpk, const float* W, const int32_t* tok,
                   const float* lse, const float* coef, float* dH, float* dW, int dw_accumulate, float* dz,
                   int64_t ldz, uint32_t* status, cudaStream_t s, int tok_base = 0, int dh_accumulate = 0);

@@ -86,6 +86,73 @@ struct FwdLseEpi {
   }
 };
 
+// FwdLseEpi that also keeps the logits for the backward (the logit store): for every 32-column
+// slice of a row, with m the running maximum after the slice (log2 units), it writes the slice's
+// e_v = 2^(x_v - m) in f16 (in (0, 1], relative precision 2^-11 down to 2^-14) through TMA and m to
+// scale[slice][row]. The sums use the same e_v, in the same order as FwdLseEpi, so lse is the same.
+// The backward turns e into dZ = coef (1[v = o] - e 2^(m - lse log2 e)) in place.
+struct FwdLseStoreEpi {
+  static constexpr bool kTmaStore = true;
+  struct Params {
+    const int32_t* tok;
+    int M, N;
+    float2* part;
+    float* ztok;
+    float* scale;   // [ceil(N / 32)][lds]
+    int64_t lds;
+  };
+  using State = FwdLseEpi::State;
+  static __device__ __forceinline__ int cols(const Params& p) { return p.N; }
+  static __device__ __forceinline__ void begin_unit(const Params& p, State& st, int row, int) {
+    st.m2 = -INFINITY;
+    st.s = 0.f;
+    st.tok = row < p.M ? __ldg(p.tok + row) : -1;
+  }
+  static __device__ __forceinline__ void chunk_to_smem(const Params& p, State& st, int row, int col0,
+                                                       const uint32_t (&r)[32], uint8_t* buf, int lane) {
+    float x[32];
+    if (col0 + 32 <= p.N) {
+#pragma unroll
+      for (int j = 0; j < 32; ++j) x[j] = __uint_as_float(r[j]) * kLog2e;
+    } else {   // the vocabulary's ragged last slice
+      const int nv = p.N - col0;
+#pragma unroll
+      for (int j = 0; j < 32; ++j) x[j] = (j < nv) ? __uint_as_float(r[j]) * kLog2e : -INFINITY;
+    }
+    float c0 = fmaxf(x[0], x[1]), c1 = fmaxf(x[2], x[3]);
+#pragma unroll
+    for (int j = 4; j < 32; j += 4) {
+      c0 = fmaxf(c0, fmaxf(x[j], x[j + 1]));
+      c1 = fmaxf(c1, fmaxf(x[j + 2], x[j + 3]));
+    }
+    const int rel = st.tok - col0;
+    if (static_cast<unsigned>(rel) < 32u) p.ztok[row] = pick32(r, rel);
+    const float mn = fmaxf(st.m2, fmaxf(c0, c1));
+#pragma unroll
+    for (int j = 0; j < 32; ++j) x[j] = ex2_ftz(x[j] - mn);
+    float a0 = 0.f, a1 = 0.f, a2 = 0.f, a3 = 0.f;
+#pragma unroll
+    for (int j = 0; j < 32; j += 4) {
+      a0 += x[j];
+      a1 += x[j + 1];
+      a2 += x[j + 2];
+      a3 += x[j + 3];
+    }
+    st.s = st.s * ex2_ftz(st.m2 - mn) + ((a0 + a1) + (a2 + a3));
+    st.m2 = mn;
+    if (row < p.M) p.scale[static_cast<int64_t>(col0 >> 5) * p.lds + row] = mn;
+    uint4* dst = reinterpret_cast<uint4*>(buf + lane * 64);
+    const int sw = (lane >> 1) & 3;
+#pragma unroll
+    for (int q = 0; q < 4; ++q)
+      dst[q ^ sw] = make_uint4(pack_f16x2(x[8 * q], x[8 * q + 1]), pack_f16x2(x[8 * q + 2], x[8 * q + 3]),
+                               pack_f16x2(x[8 * q + 4], x[8 * q + 5]), pack_f16x2(x[8 * q + 6], x[8 * q + 7]));
+  }
+  static __device__ __forceinline__ void end_unit(const Params& p, State& st, int row, int split) {
+    if (row < p.M) p.part[static_cast<size_t>(split) * p.M + row] = make_float2(st.m2, st.s);
+  }
+};
+
 // Score proxy of the cutoff design (Appendix D): besides the running max m (log2 units, over all
 // columns) keep r1 = sum_{v != o} 2^(x_v - m) and r2 = sum_{v != o} 4^(x_v - m) -- the two
 // logsumexp reductions of ||p||^2 = exp(LSE(2z) - 2 LSE(z)) with the chosen column o left out, so
@@ -332,6 +399,81 @@ struct StoreF32Epi {
   static __device__ __forceinline__ void end_unit(const Params&, State&, int, int) {}
 };
 
+// ============================================================================= logit store -> dZ
+// One block turns a 32-row x 1024-column tile of the logit store into dZ in place: the f16
+// e_v = 2^(x_v - m) of a 32-column slice (m its scale, log2 units) becomes bf16
+// dZ_v = coef (1[v = o] - p_v) with p_v = e_v 2^(m - lse log2 e), the softmax of Eq. 1's gradient
+// (Appendix D). The chosen column o takes 1 - p_o = -expm1(logp) from the forward's f32 logp
+// rather than from its f16 e, so it keeps its relative accuracy as p_o -> 1. HBM-bound: 4 bytes
+// moved per element plus 4 per 32-element slice.
+constexpr int kDzRows = 32;
+constexpr int kDzCols = 1024;
+constexpr int kDzThreads = 256;
+
+__global__ void __launch_bounds__(kDzThreads) dz_from_store_kernel(int64_t N, int V, uint16_t* z, int64_t ldz,
+                                                                   const float* scale, const int32_t* tok,
+                                                                   const float* lse, const float* logp,
+                                                                   const float* coef) {
+  __shared__ float f_s[kDzCols / 32][kDzRows];   // -coef 2^(m - lse log2 e) per slice and row
+  __shared__ float one_s[kDzRows];               // coef (1 - p_o)
+  __shared__ int tok_s[kDzRows];
+  const int64_t r0 = static_cast<int64_t>(blockIdx.x) * kDzRows;
+  const int c0 = blockIdx.y * kDzCols;
+  const int t = threadIdx.x;
+#pragma unroll
+  for (int k = 0; k < kDzCols / 32 * kDzRows / kDzThreads; ++k) {
+    const int idx = t + k * kDzThreads;
+    const int sl = idx >> 5, rr = idx & 31;
+    const int64_t row = r0 + rr;
+    const int col = c0 + sl * 32;
+    float f = 0.f;
+    if (row < N && col < V)
+      f = -__ldg(coef + row) * exp2f(__ldg(scale + static_cast<int64_t>(col >> 5) * N + row) - __ldg(lse + row) * kLog2e);
+    f_s[sl][rr] = f;
+  }
+  if (t < kDzRows) {
+    const int64_t row = r0 + t;
+    tok_s[t] = row < N ? __ldg(tok + row) : -1;
+    one_s[t] = row < N ? -__ldg(coef + row) * expm1f(__ldg(logp + row)) : 0.f;
+  }
+  __syncthreads();
+  const int warp = t >> 5, lane = t & 31;
+#pragma unroll 1
+  for (int cs = 0; cs < kDzCols; cs += 256) {
+    const int col = c0 + cs + lane * 8;   // this lane's 8 columns, inside slice col / 32
+    if (col >= V) break;
+    uint4 v[kDzRows / 8];
+#pragma unroll
+    for (int k = 0; k < kDzRows / 8; ++k) {
+      const int64_t row = r0 + warp + 8 * k;
+      if (row < N) v[k] = *reinterpret_cast<const uint4*>(z + row * ldz + col);
+    }
+#pragma unroll
+    for (int k = 0; k < kDzRows / 8; ++k) {
+      const int rr = warp + 8 * k;
+      const int64_t row = r0 + rr;
+      if (row >= N) break;
+      const float f = f_s[(cs + lane * 8) >> 5][rr];
+      const uint32_t w[4] = {v[k].x, v[k].y, v[k].z, v[k].w};
+      float o[8];
+#pragma unroll
+      for (int q = 0; q < 4; ++q) {
+        const float2 e = unpack_f16x2(w[q]);
+        o[2 * q] = e.x * f;
+        o[2 * q + 1] = e.y * f;
+      }
+      const int rel = tok_s[rr] - col;
+      if (static_cast<unsigned>(rel) < 8u) {
+#pragma unroll
+        for (int j = 0; j < 8; ++j)
+          if (j == rel) o[j] = one_s[rr];
+      }
+      *reinterpret_cast<uint4*>(z + row * ldz + col) =
+          make_uint4(pack_bf16x2(o[0], o[1]), pack_bf16x2(o[2], o[3]), pack_bf16x2(o[4], o[5]), pack_bf16x2(o[6], o[7]));
+    }
+  }
+}
+
 // ============================================================================= host side
 typedef CUresult (*EncodeTiledFn)(CUtensorMap*, CUtensorMapDataType, cuuint32_t, void*, const cuuint64_t*,
                                   const cuuint64_t*, const cuuint32_t*, const cuuint32_t*, CUtensorMapInterleave,
@@ -351,10 +493,12 @@ static EncodeTiledFn encode_fn() {
   return fn;
 }
 
-// 2-D bf16 tensor [outer][inner] with row pitch `pitch_bytes`, 128-byte swizzled boxes.
+// 2-D tensor of 2-byte elements (bf16 unless `type` says f16) [outer][inner] with row pitch
+// `pitch_bytes`, 128-byte swizzled boxes unless `swizzle` says otherwise.
 static bool make_map(CUtensorMap* m, const void* base, uint64_t inner, uint64_t outer, uint64_t pitch_bytes,
                      uint32_t box_inner, uint32_t box_outer,
-                     CUtensorMapSwizzle swizzle = CU_TENSOR_MAP_SWIZZLE_128B) {
+                     CUtensorMapSwizzle swizzle = CU_TENSOR_MAP_SWIZZLE_128B,
+                     CUtensorMapDataType type = CU_TENSOR_MAP_DATA_TYPE_BFLOAT16) {
   EncodeTiledFn enc = encode_fn();
   if (!enc) return false;
   if ((reinterpret_cast<uintptr_t>(base) & 15) || (pitch_bytes & 15)) return false;
@@ -362,7 +506,7 @@ static bool make_map(CUtensorMap* m, const void* base, uint64_t inner, uint64_t 
   const cuuint64_t strides[1] = {pitch_bytes};
   const cuuint32_t box[2] = {box_inner, box_outer};
   const cuuint32_t estr[2] = {1, 1};
-  return enc(m, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<void*>(base), dims, strides, box, estr,
+  return enc(m, type, 2, const_cast<void*>(base), dims, strides, box, estr,
              CU_TENSOR_MAP_INTERLEAVE_NONE, swizzle, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
              CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
 }
@@ -525,6 +669,24 @@ int fwd_gemm_bf16(int64_t N, int d, int V, const void* Hpk, const void* W, const
   return launch_gemm_single<false, false, FwdLseEpi, 2>(ta, tb, ta, N, V, d, splits, band, ep, status, s);
 }
 
+// The forward that keeps its logits: f16 e [N][ldz] through TMA (32 x 32 boxes from 64-byte-swizzled
+// staging) and the slice maxima scale [ceil(V / 32)][N].
+int fwd_gemm_store_bf16(int64_t N, int d, int V, const void* Hpk, const void* W, const int32_t* tok, float2* part,
+                        float* ztok, int splits, void* store, int64_t ldz, float* scale, uint32_t* status,
+                        cudaStream_t s) {
+  const int halves = fwd_halves(d);
+  CUtensorMap ta, tb, tc;
+  if (!map_kmajor(&ta, Hpk, N, d, d, kBM * halves) || !map_kmajor(&tb, W, V, d, d, kBRowsBox)) return PS_ERR_INVALID_ARG;
+  if (!make_map(&tc, store, V, N, ldz * 2, 32, 32, CU_TENSOR_MAP_SWIZZLE_64B, CU_TENSOR_MAP_DATA_TYPE_FLOAT16))
+    return PS_ERR_INVALID_ARG;
+  FwdLseStoreEpi::Params ep{tok, static_cast<int>(N), V, part, ztok, scale, N};
+  const int workers = num_sms_current();
+  const int band = splits == fwd_tile_splits_bf16(V) ? fwd_band_max(d) : (workers + splits - 1) / splits;
+  if (halves == 1)
+    return launch_gemm_single<false, false, FwdLseStoreEpi, 1>(ta, tb, tc, N, V, d, splits, band, ep, status, s);
+  return launch_gemm_single<false, false, FwdLseStoreEpi, 2>(ta, tb, tc, N, V, d, splits, band, ep, status, s);
+}
+
 // Bands (row blocks walked together) of the backward GEMMs. Recompute: 32 row blocks of 128 rows
 // (16 of its 256-row tiles) share each W tile; their hidden rows, 29 MB at d = 3584, stay in L2
 // beside the W tiles in flight and the streamed dZ (44 MB bands read 46% more DRAM). dH and dW: bands of 4 row
@@ -577,8 +739,15 @@ int bwd_chunk_bf16(int64_t rc, int d, int V, const void* Hpk, const void* W, con
                                                                     kBandRecompute / kRecHalves, ep, status, s);
     if (rcode != PS_OK) return rcode;
   }
-  // dH (K = V) and dW (K = chunk rows) have long K loops: one CTA computes a 256 x 256 tile
-  // as two M = 128 halves that share each B stage (a third fewer operand bytes per FLOP).
+  return bwd_grads_bf16(rc, d, V, Hpk, W, dH, dW, dw_accumulate, dz, ldz, status, s, dh_accumulate);
+}
+
+// dH = dZ W and dW (+)= dZ^T H over rc rows of dZ [rc][ldz] bf16. Both have long K loops (V and rc):
+// one CTA computes a 256 x 256 tile as two M = 128 halves that share each B stage (a third fewer
+// operand bytes per FLOP).
+int bwd_grads_bf16(int64_t rc, int d, int V, const void* Hpk, const void* W, float* dH, float* dW, int dw_accumulate,
+                   const void* dz, int64_t ldz, uint32_t* status, cudaStream_t s, int dh_accumulate) {
+  int rcode;
   if (dH) {
     CUtensorMap ta, tb;
     if (!map_kmajor(&ta, dz, rc, V, ldz, 2 * kBM) || !map_mnmajor(&tb, W, V, d, d)) return PS_ERR_INVALID_ARG;
@@ -594,6 +763,15 @@ int bwd_chunk_bf16(int64_t rc, int d, int V, const void* Hpk, const void* W, con
     if (rcode != PS_OK) return rcode;
   }
   return PS_OK;
+}
+
+int dz_from_store_bf16(int64_t N, int V, void* store, int64_t ldz, const float* scale, const int32_t* tok,
+                       const float* lse, const float* logp, const float* coef, cudaStream_t s) {
+  if (N == 0) return PS_OK;
+  const dim3 grid(static_cast<unsigned>((N + kDzRows - 1) / kDzRows), static_cast<unsigned>((V + kDzCols - 1) / kDzCols));
+  dz_from_store_kernel<<<grid, kDzThreads, 0, s>>>(N, V, static_cast<uint16_t*>(store), ldz, scale, tok, lse, logp,
+                                                   coef);
+  return cudaGetLastError() == cudaSuccess ? PS_OK : PS_ERR_CUDA;
 }
 
 int gemm_bf16(int M, int N, int K, int a_mn, int b_mn, const void* A, int64_t lda, const void* B, int64_t ldb,

@@ -259,6 +259,21 @@ __device__ __forceinline__ uint32_t pack_bf16x2(float lo, float hi) {
   return r;
 }
 
+__device__ __forceinline__ uint32_t pack_f16x2(float lo, float hi) {
+  uint32_t r;
+  asm("cvt.rn.f16x2.f32 %0, %1, %2;" : "=r"(r) : "f"(hi), "f"(lo));
+  return r;
+}
+
+// The two f16 halves of a 32-bit word as floats (low half first).
+__device__ __forceinline__ float2 unpack_f16x2(uint32_t v) {
+  unsigned short lo = static_cast<unsigned short>(v & 0xffffu), hi = static_cast<unsigned short>(v >> 16);
+  float a, b;
+  asm("cvt.f32.f16 %0, %1;" : "=f"(a) : "h"(lo));
+  asm("cvt.f32.f16 %0, %1;" : "=f"(b) : "h"(hi));
+  return make_float2(a, b);
+}
+
 // ================================================================== philox4x64-10
 // Salmon et al., "Parallel Random Numbers: As Easy as 1, 2, 3" (SC'11).
 __device__ __forceinline__ void philox4x64_10(uint64_t (&c)[4], uint64_t k0, uint64_t k1) {

@@ -600,16 +600,37 @@ size_t ps_lmhead_ppo_fwd_workspace_size(int64_t N, int d, int V, int dtype) {
   return fwd_ws(nullptr, N, V, dtype, SIZE_MAX).bytes;
 }
 
-int ps_lmhead_ppo_fwd(int64_t N, int d, int V, int dtype, const void* Hpk, const void* W, const int32_t* tok,
-                      const float* oldlogp, const float* adv, const float* w, double eps, double loss_scale,
-                      double* loss, float* lse, float* logp, float* ratio, float* coef, float* row_loss, void* ws,
-                      size_t ws_bytes, ps_stream_t stream) {
-  NvtxRange nvtx_range("ps_lmhead_ppo_fwd");
+}  // extern "C"
+
+// Layout of the logit store of N rows: [N][ldz] 2-byte values (f16 e after the forward, bf16 dZ after
+// the backward's conversion), then the slice maxima [ceil(V / 32)][N] f32 at a 256-byte boundary.
+struct StoreLayout {
+  int64_t ldz;
+  size_t scale_off;
+  size_t bytes;
+};
+static StoreLayout store_layout(int64_t N, int V) {
+  StoreLayout L;
+  L.ldz = ldz_for(V);
+  L.scale_off = align_up(static_cast<size_t>(N) * static_cast<size_t>(L.ldz) * 2, 256);
+  L.bytes = L.scale_off + sizeof(float) * static_cast<size_t>((V + 31) / 32) * static_cast<size_t>(N);
+  return L;
+}
+
+static int lmhead_fwd_impl(int64_t N, int d, int V, int dtype, const void* Hpk, const void* W, const int32_t* tok,
+                           const float* oldlogp, const float* adv, const float* w, double eps, double loss_scale,
+                           double* loss, float* lse, float* logp, float* ratio, float* coef, float* row_loss,
+                           void* store, size_t store_bytes, void* ws, size_t ws_bytes, ps_stream_t stream) {
   if (N < 0 || N > INT32_MAX || V < 1 || !dtype_ok(dtype) || !d_ok(d, dtype)) return PS_ERR_INVALID_ARG;
   if (!(eps >= 0.0) || !loss || (N > 0 && (!Hpk || !W || !tok || !oldlogp || !adv || !w || !lse || !logp ||
                                            !ratio || !coef)))
     return PS_ERR_INVALID_ARG;
   if (N > 0 && (!al16(Hpk) || !al16(W))) return PS_ERR_INVALID_ARG;
+  if (store != nullptr) {
+    if (dtype != PS_DTYPE_BF16) return PS_ERR_UNSUPPORTED;
+    if (!al16(store)) return PS_ERR_INVALID_ARG;
+    if (store_bytes < store_layout(N, V).bytes) return PS_ERR_WORKSPACE;
+  }
   if (dtype == PS_DTYPE_BF16 && !device_is_sm103()) return PS_ERR_UNSUPPORTED;
   cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
   FwdWs f = fwd_ws(ws, N, V, dtype, ws_bytes);
@@ -620,7 +641,13 @@ int ps_lmhead_ppo_fwd(int64_t N, int d, int V, int dtype, const void* Hpk, const
   int splits;
   if (dtype == PS_DTYPE_BF16) {
     splits = choose_fwd_splits_bf16(N, d, V, num_sms_current(), f.splits);
-    rc = fwd_gemm_bf16(N, d, V, Hpk, W, tok, f.part, f.ztok, splits, status_word(ws), s);
+    if (store) {
+      const StoreLayout L = store_layout(N, V);
+      float* scale = reinterpret_cast<float*>(static_cast<uint8_t*>(store) + L.scale_off);
+      rc = fwd_gemm_store_bf16(N, d, V, Hpk, W, tok, f.part, f.ztok, splits, store, L.ldz, scale, status_word(ws), s);
+    } else {
+      rc = fwd_gemm_bf16(N, d, V, Hpk, W, tok, f.part, f.ztok, splits, status_word(ws), s);
+    }
   } else {
     splits = fwd_splits_f32(V);
     rc = fwd_gemm_f32(N, d, V, static_cast<const float*>(Hpk), static_cast<const float*>(W), tok, f.part, f.ztok,
@@ -634,6 +661,64 @@ int ps_lmhead_ppo_fwd(int64_t N, int d, int V, int dtype, const void* Hpk, const
   if (cudaGetLastError() != cudaSuccess) return PS_ERR_CUDA;
   loss_reduce_kernel<<<1, 1024, 0, s>>>(nb, f.block_loss, loss);
   return cudaGetLastError() == cudaSuccess ? PS_OK : PS_ERR_CUDA;
+}
+
+extern "C" {
+
+int ps_lmhead_ppo_fwd(int64_t N, int d, int V, int dtype, const void* Hpk, const void* W, const int32_t* tok,
+                      const float* oldlogp, const float* adv, const float* w, double eps, double loss_scale,
+                      double* loss, float* lse, float* logp, float* ratio, float* coef, float* row_loss, void* ws,
+                      size_t ws_bytes, ps_stream_t stream) {
+  NvtxRange nvtx_range("ps_lmhead_ppo_fwd");
+  return lmhead_fwd_impl(N, d, V, dtype, Hpk, W, tok, oldlogp, adv, w, eps, loss_scale, loss, lse, logp, ratio, coef,
+                         row_loss, nullptr, 0, ws, ws_bytes, stream);
+}
+
+size_t ps_lmhead_logit_store_size(int64_t N, int V) {
+  if (N < 0 || N > INT32_MAX || V < 1) return 0;
+  return store_layout(N, V).bytes;
+}
+
+int ps_lmhead_ppo_fwd_store(int64_t N, int d, int V, int dtype, const void* Hpk, const void* W, const int32_t* tok,
+                            const float* oldlogp, const float* adv, const float* w, double eps, double loss_scale,
+                            double* loss, float* lse, float* logp, float* ratio, float* coef, float* row_loss,
+                            void* store, size_t store_bytes, void* ws, size_t ws_bytes, ps_stream_t stream) {
+  NvtxRange nvtx_range("ps_lmhead_ppo_fwd_store");
+  if (store == nullptr) return PS_ERR_INVALID_ARG;
+  return lmhead_fwd_impl(N, d, V, dtype, Hpk, W, tok, oldlogp, adv, w, eps, loss_scale, loss, lse, logp, ratio, coef,
+                         row_loss, store, store_bytes, ws, ws_bytes, stream);
+}
+
+size_t ps_lmhead_ppo_bwd_from_store_workspace_size(void) { return kWsHeader; }
+
+int ps_lmhead_ppo_bwd_from_store(int64_t N, int d, int V, int dtype, const void* Hpk, const void* W,
+                                 const int32_t* tok, const float* lse, const float* logp, const float* coef,
+                                 void* store, size_t store_bytes, float* dH, float* dW, int flags, void* ws,
+                                 size_t ws_bytes, ps_stream_t stream) {
+  NvtxRange nvtx_range("ps_lmhead_ppo_bwd_from_store");
+  if (N < 0 || N > INT32_MAX || V < 1 || !dtype_ok(dtype) || !d_ok(d, dtype)) return PS_ERR_INVALID_ARG;
+  if (flags & ~(PS_DW_ACCUMULATE | PS_DH_ACCUMULATE)) return PS_ERR_INVALID_ARG;
+  if (dtype != PS_DTYPE_BF16) return PS_ERR_UNSUPPORTED;
+  if (N > 0 && (!Hpk || !W || !tok || !lse || !logp || !coef || !store)) return PS_ERR_INVALID_ARG;
+  if ((N > 0 && (!al16(Hpk) || !al16(W) || !al16(store))) || (dH && !al16(dH)) || (dW && !al16(dW)))
+    return PS_ERR_INVALID_ARG;
+  if (N > 0 && store_bytes < store_layout(N, V).bytes) return PS_ERR_WORKSPACE;
+  if (!device_is_sm103()) return PS_ERR_UNSUPPORTED;
+  cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
+  int rc = begin_call(ws, ws_bytes, kWsHeader, s);
+  if (rc != PS_OK) return rc;
+  if (N == 0) {
+    if (dW && !(flags & PS_DW_ACCUMULATE))
+      return cudaMemsetAsync(dW, 0, sizeof(float) * static_cast<size_t>(V) * d, s) == cudaSuccess ? PS_OK
+                                                                                                : PS_ERR_CUDA;
+    return PS_OK;
+  }
+  const StoreLayout L = store_layout(N, V);
+  const float* scale = reinterpret_cast<const float*>(static_cast<const uint8_t*>(store) + L.scale_off);
+  rc = dz_from_store_bf16(N, V, store, L.ldz, scale, tok, lse, logp, coef, s);
+  if (rc != PS_OK) return rc;
+  return bwd_grads_bf16(N, d, V, Hpk, W, dH, dW, (flags & PS_DW_ACCUMULATE) ? 1 : 0, store, L.ldz, status_word(ws), s,
+                        (flags & PS_DH_ACCUMULATE) ? 1 : 0);
 }
 
 size_t ps_lmhead_logit_stats_workspace_size(int64_t N, int d, int Vs, int dtype) {

@@ -2,7 +2,9 @@
 
 UpdatePass owns the device buffers of one batch shape (allocated once with torch,
 sized for the worst case N = sum L) and runs the four library calls in order on the
-current stream: cutoffs -> packed prefixes -> fused forward -> fused backward.
+current stream: cutoffs -> packed prefixes -> fused forward -> fused backward. With a
+logit store (PassShape.store_rows), a step whose N fits keeps the forward's logits for
+the backward instead of recomputing them.
 The only host synchronisation is reading N after packing.
 CutoffDesign does the same for the cutoff design upstream of the update (score
 proxy and top-k next tokens, u_t, and the design into sampler masses).
@@ -29,6 +31,8 @@ class PassShape:
     capacity: int                 # max packed rows (sum of lengths)
     dtype: torch.dtype = torch.bfloat16
     bwd_chunk_rows: int = 32768   # rows of dZ held at once in the backward workspace
+    store_rows: int = 0           # rows of the logit store (bf16): a step with N <= store_rows keeps
+                                  # its logits from the forward instead of recomputing them (0: never)
 
 
 class UpdatePass:
@@ -67,7 +71,14 @@ class UpdatePass:
         self.ws_fwd = torch.zeros(B.ps_lmhead_ppo_fwd_workspace_size(cap, s.d, s.V, self.dcode), **u8)
         self.ws_bwd = torch.zeros(B.ps_lmhead_ppo_bwd_workspace_size(cap, s.d, s.V, self.dcode,
                                                                      min(s.bwd_chunk_rows, cap)), **u8)
+        self.store = None
+        if s.store_rows > 0:
+            if s.dtype != torch.bfloat16:
+                raise ValueError("the logit store needs a bf16 head")
+            self.store = torch.empty(B.ps_lmhead_logit_store_size(min(s.store_rows, cap), s.V), **u8)
         self.N = 0
+        self.use_store = True         # False: recompute even where the store would hold the step
+        self.stored = False           # the last forward filled the store (its backward reads it)
 
     def sample(self, q, L, seed, step, traj_base=0):
         s = self.s
@@ -84,14 +95,27 @@ class UpdatePass:
 
     def forward(self, W):
         s = self.s
-        B.ps_lmhead_ppo_fwd(self.N, s.d, s.V, self.dcode, self.hid, W, self.tok, self.oldlogp, self.adv, self.w,
-                            self.eps, self.loss_scale, self.loss, self.lse, self.logp, self.ratio, self.coef,
-                            self.row_loss, self.ws_fwd)
+        self.stored = self.use_store and self.store is not None and self.N <= s.store_rows
+        if self.stored:
+            B.ps_lmhead_ppo_fwd_store(self.N, s.d, s.V, self.dcode, self.hid, W, self.tok, self.oldlogp, self.adv,
+                                      self.w, self.eps, self.loss_scale, self.loss, self.lse, self.logp, self.ratio,
+                                      self.coef, self.row_loss, self.store, self.ws_fwd)
+        else:
+            B.ps_lmhead_ppo_fwd(self.N, s.d, s.V, self.dcode, self.hid, W, self.tok, self.oldlogp, self.adv, self.w,
+                                self.eps, self.loss_scale, self.loss, self.lse, self.logp, self.ratio, self.coef,
+                                self.row_loss, self.ws_fwd)
 
     def backward(self, W, dw_accumulate: bool = False):
         s = self.s
-        B.ps_lmhead_ppo_bwd(self.N, s.d, s.V, self.dcode, self.hid, W, self.tok, self.lse, self.coef, self.dH,
-                            self.dW, B.PS_DW_ACCUMULATE if dw_accumulate else B.PS_DW_OVERWRITE, self.ws_bwd)
+        flags = B.PS_DW_ACCUMULATE if dw_accumulate else B.PS_DW_OVERWRITE
+        if self.stored:
+            # the store turns into dZ in place: one backward per forward
+            self.stored = False
+            B.ps_lmhead_ppo_bwd_from_store(self.N, s.d, s.V, self.dcode, self.hid, W, self.tok, self.lse, self.logp,
+                                           self.coef, self.store, self.dH, self.dW, flags, self.ws_bwd)
+        else:
+            B.ps_lmhead_ppo_bwd(self.N, s.d, s.V, self.dcode, self.hid, W, self.tok, self.lse, self.coef, self.dH,
+                                self.dW, flags, self.ws_bwd)
 
     def run(self, q, L, R, tok_full, oldlogp_full, hid_full, W, seed, step, traj_base=0, grads=True) -> int:
         self.sample(q, L, seed, step, traj_base)

@@ -86,7 +86,7 @@ def maxrel(a, b):
 # launch changes hands: the backward's chunking (csrc/psppo_api.cu) and the row bands of the
 # forward, recompute and dH/dW GEMMs (csrc/lmhead_bf16.cu).
 FWD_BAND_L2_BYTES = 30e6      # hidden rows of one forward band
-REC_BAND_BLOCKS = 48          # 128-row blocks per recompute band
+REC_BAND_BLOCKS = 32          # 128-row blocks per recompute band
 GRAD_BAND_ROWS = 4 * 256      # dH / dW bands: 4 tiles of 256 rows
 
 

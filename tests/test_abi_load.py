@@ -126,3 +126,35 @@ def test_vocabulary_shard_arguments_are_rejected_on_the_host(lib):
     assert bwd(10, 0, 0, 1024) == INV
     assert L.ps_lmhead_logit_stats_workspace_size(10, 128, 64, 0) == L.ps_lmhead_ppo_fwd_workspace_size(10, 128, 64, 0)
     assert L.ps_lmhead_ppo_fwd_from_stats_workspace_size(1000) >= 256 + 8 * 4
+
+
+def test_logit_store_layout_and_refusals_on_the_host(lib):
+    # The store's size is its layout: [N][ldz] 2-byte values, ldz = V rounded up to 8, then the f32 slice
+    # maxima [ceil(V/32)][N] from the next 256-byte boundary. Bad arguments fail before any CUDA call.
+    import ctypes
+    L = lib
+    INV, UNSUP, WS = 1, 2, 3
+    assert L.ps_lmhead_logit_store_size(1000, 152064) == 1000 * 152064 * 2 + 4 * 4752 * 1000
+    assert L.ps_lmhead_logit_store_size(3, 1001) == 6144 + 4 * 32 * 3          # 3 x 1008 x 2 = 6048 -> 6144
+    assert L.ps_lmhead_logit_store_size(0, 1024) == 0
+    assert L.ps_lmhead_logit_store_size(-1, 1024) == 0 and L.ps_lmhead_logit_store_size(10, 0) == 0
+    assert L.ps_lmhead_ppo_bwd_from_store_workspace_size() == 256
+    fake = ctypes.c_void_p(1 << 20)     # 16-byte aligned, never dereferenced: the checks fail first
+    p = (fake,) * 6
+
+    def fwd(dt, store, nbytes, d=128, V=1024):
+        return L.ps_lmhead_ppo_fwd_store(10, d, V, dt, *p, 0.2, 1.0, fake, fake, fake, fake, fake, None, store,
+                                         nbytes, None, 0, None)
+    need = L.ps_lmhead_logit_store_size(10, 1024)
+    assert fwd(0, None, need) == INV                              # no store
+    assert fwd(1, fake, need) == UNSUP                            # f32 head: recompute only
+    assert fwd(0, ctypes.c_void_p((1 << 20) + 8), need) == INV    # misaligned store
+    assert fwd(0, fake, need - 1) == WS                           # too small
+    assert fwd(0, fake, need, d=100) == INV
+
+    def bwd(dt, store, nbytes, flags=0):
+        return L.ps_lmhead_ppo_bwd_from_store(10, 128, 1024, dt, *p, store, nbytes, fake, fake, flags, None, 0, None)
+    assert bwd(1, fake, need) == UNSUP
+    assert bwd(0, None, need) == INV
+    assert bwd(0, fake, need, flags=4) == INV                     # unknown flag
+    assert bwd(0, fake, need - 1) == WS
