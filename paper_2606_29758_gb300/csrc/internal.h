@@ -46,9 +46,10 @@ int bwd_chunk_bf16(int64_t rc, int d, int V, const void* Hpk, const void* W, con
 // dH = dZ W and dW (+)= dZ^T Hpk from dZ [rc][ldz] bf16 already in memory.
 int bwd_grads_bf16(int64_t rc, int d, int V, const void* Hpk, const void* W, float* dH, float* dW, int dw_accumulate,
                    const void* dz, int64_t ldz, uint32_t* status, cudaStream_t s, int dh_accumulate);
-// The logit store of the forward turned into dZ in place (f16 e -> bf16 dZ), rows [0, N).
-int dz_from_store_bf16(int64_t N, int V, void* store, int64_t ldz, const float* scale, const int32_t* tok,
-                       const float* lse, const float* logp, const float* coef, cudaStream_t s);
+// The logit store of the forward turned into dZ in place (f16 e -> bf16 dZ), rows [0, N) of already
+// offset pointers; scale [c][lds] (lds: the store's row count, the pitch of its slice maxima).
+int dz_from_store_bf16(int64_t N, int V, void* store, int64_t ldz, const float* scale, int64_t lds,
+                       const int32_t* tok, const float* lse, const float* logp, const float* coef, cudaStream_t s);
 int bwd_chunk_f32(int64_t rc, int d, int V, const float* Hpk, const float* W, const int32_t* tok,
                   const float* lse, const float* coef, float* dH, float* dW, int dw_accumulate, float* dz,
                   int64_t ldz, uint32_t* status, cudaStream_t s, int tok_base = 0, int dh_accumulate = 0);

@@ -71,6 +71,8 @@ CONFIGS["head1.5b_small"] = Config("head1.5b_small", P=1, K=4, len_law="uniform"
 CONFIGS["mid_f32"] = replace(CONFIGS["mid"], name="mid_f32", dtype="f32")
 # The 7B-shaped head on two prompts (about 25k packed rows): a small case for profiling.
 CONFIGS["7b_p2"] = replace(CONFIGS["7b"], name="7b_p2", P=2)
+# The 7B-shaped head on one group of four (about 7k packed rows): a capture of a few GB of device memory.
+CONFIGS["7b_p1k4"] = replace(CONFIGS["7b"], name="7b_p1k4", P=1, K=4)
 
 
 def get_config(name: str, **overrides) -> Config:

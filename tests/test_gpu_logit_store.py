@@ -224,12 +224,12 @@ def test_store_with_no_rows():
     assert loss.item() == 0.0 and float(dW.abs().max()) == 0.0
 
 
-def test_store_at_the_7b_workload():
-    # the benchmark's 7B workload through the store path: the forward bit-identical to the recompute
-    # path's; dH on a stratified set of rows (every 128-row block, the forward's band edges, the dH
-    # bands and the last tile) and dZ on 96 of them against the oracle; sum_v dW = 0; dW against the
-    # recompute path's
-    cfg = get_config("7b")
+@pytest.mark.parametrize("name", ["7b", "1.5b"])
+def test_store_at_full_size(name):
+    # a full-size workload through the store path: the forward bit-identical to the recompute path's; dH on a stratified set of rows (every 128-row block, the forward's band edges,
+    # the dH bands and the last tile) and dZ on about 96 of them against the oracle; sum_v dW = 0; dW
+    # against the recompute path's
+    cfg = get_config(name)
     b = make_batch(cfg, device="cuda")
     D = b.dev
     rec, sto = _two_passes(cfg, b)
@@ -269,6 +269,6 @@ def test_store_at_the_7b_workload():
     bound = (sto.coef[:N].abs()[:, None] * sto.hid[:N].float().abs()).double().sum(dim=0) * 2.0 ** -8
     assert (colsum.abs() / (1.5 * bound + 1e-6 * sto.dW.abs().max().double())).max().item() < 1.0
     err_w = (sto.dW - rec.dW).abs().max().item() / rec.dW.abs().max().item()
-    print("7b", N, "rows", len(rows), "dH max-rel", err_h, "dZ worst / bound", worst, "dW store vs recompute", err_w)
+    print(name, N, "rows", len(rows), "dH max-rel", err_h, "dZ worst / bound", worst, "dW store vs recompute", err_w)
     assert err_w < 1e-2
     assert torch.isfinite(sto.dW).all() and torch.isfinite(sto.dH[:N]).all()
