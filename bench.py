@@ -44,9 +44,10 @@ MEASURED_PEAKS = os.path.join(ROOT, "MEASURED_PEAKS.json")
 FALLBACK_PEAKS = {"hbm_gbs": 6800.0, "bf16_tflops": 1900.0, "bf16_tflops_sustained": 1700.0}
 
 # DRAM bytes (read + write) per launch of the forward GEMM on the 7b workload, the mean of the
-# six launches in profiles/lmhead_pass_7b_launch_list.md (55.39 GB read + 0.92 GB written).
-# Reset to None whenever the forward kernel or its schedule changes.
-FWD_GEMM_TRAFFIC = {("7b", "FwdLseEpi"): 56.31e9}
+# launches in profiles/lmhead_pass_7b_launch_list.md: the plain forward 55.39 GB read + 0.92 GB
+# written, the forward keeping its logits 53.69 GB read + 63.26 GB written (its algorithmic write is
+# the logit store, 64.5 GB). Reset an entry whenever that kernel or its schedule changes.
+FWD_GEMM_TRAFFIC = {("7b", "FwdLseEpi"): 56.31e9, ("7b", "FwdLseStoreEpi"): 116.95e9}
 
 
 def describe(cfg) -> str:
@@ -136,9 +137,16 @@ def logit_store_rows(args, cfg, b, dev):
     if args.logits == "recompute" or cfg.dtype != "bf16":
         return 0
     free, _ = torch.cuda.mem_get_info(dev)
-    other = 40e9 + b.total_len * cfg.d * 12.0 + cfg.V * cfg.d * 8.0 + args.chunk_rows * cfg.V * 2.0
-    per_row = ps_lmhead_logit_store_size(1 << 16, cfg.V) / (1 << 16)
-    return int(max(0, min(b.total_len, (free - other) // per_row)))
+    rows, d, V = b.total_len, cfg.d, cfg.V
+    other = (rows * d * 6.0                          # packed hidden rows (bf16) and dH (f32)
+             + rows * ((V + 255) // 256 * 8.0 + 64)  # forward partials, per-row vectors
+             + min(args.chunk_rows, rows) * V * 2.0  # the recompute path's dZ chunk
+             + V * d * 4.0                           # dW
+             + rows * (d * 4.0 + 32)                 # the end-to-end stager's two input buffers
+             + rows * 3e3                            # the design stage's proxy and top-16 buffers
+             + 20e9)                                 # margin
+    per_row = ps_lmhead_logit_store_size(1 << 16, V) / (1 << 16)
+    return int(max(0, min(rows, (free - other) // per_row)))
 
 
 def run_ours(args):
