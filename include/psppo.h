@@ -289,6 +289,27 @@ int ps_lmhead_ppo_bwd_vocab_shard(int64_t N, int d, int Vs, int64_t v0, int V, i
                                   const float* lse, const float* coef, float* dH, float* dW_shard,
                                   int flags, void* ws, size_t ws_bytes, ps_stream_t stream);
 
+/* The vocabulary-parallel steps with a logit store per shard (bf16 only):
+ * ps_lmhead_logit_stats_store: ps_lmhead_logit_stats (same arguments, outputs, workspace and
+ *   errors) that also fills the shard's store, laid out as for ps_lmhead_ppo_fwd_store with
+ *   Vs columns (store_bytes >= ps_lmhead_logit_store_size(N, Vs), else PS_ERR_WORKSPACE).
+ * ps_lmhead_ppo_bwd_vocab_shard_from_store: ps_lmhead_ppo_bwd_vocab_shard from the shard's
+ *   store, which it overwrites with the shard's dZ [N][ldz] (ldz = Vs rounded up to 8), as
+ *   ps_lmhead_ppo_bwd_from_store does; lse, logp and coef from step 3 (the one-hot column
+ *   takes 1 - exp(logp_i) where tok_i - v0 is in [0, Vs)). Workspace: the status header,
+ *   ps_lmhead_ppo_bwd_from_store_workspace_size() bytes.
+ */
+int ps_lmhead_logit_stats_store(int64_t N, int d, int Vs, int64_t v0, int dtype, const void* Hpk,
+                                const void* W_shard, const int32_t* tok, float* stats, float* ztok,
+                                void* store, size_t store_bytes, void* ws, size_t ws_bytes,
+                                ps_stream_t stream);
+int ps_lmhead_ppo_bwd_vocab_shard_from_store(int64_t N, int d, int Vs, int64_t v0, int V, int dtype,
+                                             const void* Hpk, const void* W_shard, const int32_t* tok,
+                                             const float* lse, const float* logp, const float* coef,
+                                             void* store, size_t store_bytes, float* dH,
+                                             float* dW_shard, int flags, void* ws, size_t ws_bytes,
+                                             ps_stream_t stream);
+
 /* ---------------------------------------------------------------------------
  * ps_lmhead_score_proxy -- per-token output-head score proxy (cutoff design input).
  *

@@ -32,7 +32,7 @@ EXPORTS = [
     "ps_lmhead_logit_stats_workspace_size", "ps_lmhead_logit_stats",
     "ps_lmhead_ppo_fwd_from_stats_workspace_size", "ps_lmhead_ppo_fwd_from_stats", "ps_lmhead_ppo_bwd_vocab_shard",
     "ps_lmhead_logit_store_size", "ps_lmhead_ppo_fwd_store", "ps_lmhead_ppo_bwd_from_store_workspace_size",
-    "ps_lmhead_ppo_bwd_from_store",
+    "ps_lmhead_ppo_bwd_from_store", "ps_lmhead_logit_stats_store", "ps_lmhead_ppo_bwd_vocab_shard_from_store",
     "ps_diag_gemm_bf16", "ps_diag_wait_timeout", "ps_lmhead_ppo_fwd_noalloc",
     "ps_lmhead_score_proxy_workspace_size", "ps_lmhead_score_proxy",
     "ps_design_cutoffs_workspace_size", "ps_design_cutoffs",
@@ -91,6 +91,10 @@ _SIGS = {
     "ps_lmhead_ppo_bwd_from_store_workspace_size": (_sz, []),
     "ps_lmhead_ppo_bwd_from_store": (_i32, [_i64, _i32, _i32, _i32, _vp, _vp, _vp, _vp, _vp, _vp, _vp, _sz, _vp, _vp,
                                             _i32, _vp, _sz, _vp]),
+    "ps_lmhead_logit_stats_store": (_i32, [_i64, _i32, _i32, _i64, _i32, _vp, _vp, _vp, _vp, _vp, _vp, _sz, _vp, _sz,
+                                           _vp]),
+    "ps_lmhead_ppo_bwd_vocab_shard_from_store": (_i32, [_i64, _i32, _i32, _i64, _i32, _i32, _vp, _vp, _vp, _vp, _vp,
+                                                        _vp, _vp, _sz, _vp, _vp, _i32, _vp, _sz, _vp]),
     "ps_diag_gemm_bf16": (_i32, [_i32, _i32, _i32, _i32, _i32, _vp, _i64, _vp, _i64, _vp, _i64, _i32, _i32, _vp, _sz,
                                  _vp]),
     "ps_diag_wait_timeout": (_i32, [_u64, _vp, _sz, _vp]),
@@ -322,6 +326,22 @@ def ps_lmhead_ppo_bwd_from_store(N, d, V, dtype, Hpk, W, tok, lse, logp, coef, s
                                             _ptr(coef), _ptr(store), _nbytes(store), _ptr(dH), _ptr(dW), flags,
                                             _ptr(ws), _nbytes(ws), _stream(stream))
     _check(rc, "ps_lmhead_ppo_bwd_from_store")
+
+
+def ps_lmhead_logit_stats_store(N, d, Vs, v0, dtype, Hpk, W_shard, tok, stats, ztok, store, ws, stream=None):
+    rc = lib().ps_lmhead_logit_stats_store(N, d, Vs, v0, dtype, _ptr(Hpk), _ptr(W_shard), _ptr(tok), _ptr(stats),
+                                           _ptr(ztok), _ptr(store), _nbytes(store), _ptr(ws), _nbytes(ws),
+                                           _stream(stream))
+    _check(rc, "ps_lmhead_logit_stats_store")
+
+
+def ps_lmhead_ppo_bwd_vocab_shard_from_store(N, d, Vs, v0, V, dtype, Hpk, W_shard, tok, lse, logp, coef, store, dH,
+                                             dW_shard, flags, ws, stream=None):
+    rc = lib().ps_lmhead_ppo_bwd_vocab_shard_from_store(N, d, Vs, v0, V, dtype, _ptr(Hpk), _ptr(W_shard), _ptr(tok),
+                                                        _ptr(lse), _ptr(logp), _ptr(coef), _ptr(store),
+                                                        _nbytes(store), _ptr(dH), _ptr(dW_shard), flags, _ptr(ws),
+                                                        _nbytes(ws), _stream(stream))
+    _check(rc, "ps_lmhead_ppo_bwd_vocab_shard_from_store")
 
 
 def ps_diag_gemm_bf16(M, N, K, a_mn_major, b_mn_major, A, lda, B, ldb, C, ldc, accumulate, ws, variant=0,

@@ -22,7 +22,7 @@ int fwd_gemm_bf16(int64_t N, int d, int V, const void* Hpk, const void* W, const
 // 32-column slice, m the running row maximum after the slice (log2 units), in scale [ceil(V/32)][N].
 int fwd_gemm_store_bf16(int64_t N, int d, int V, const void* Hpk, const void* W, const int32_t* tok, float2* part,
                         float* ztok, int splits, void* store, int64_t ldz, float* scale, uint32_t* status,
-                        cudaStream_t s);
+                        cudaStream_t s, int tok_base = 0);
 int fwd_splits_f32(int V);
 int fwd_gemm_f32(int64_t N, int d, int V, const float* Hpk, const float* W, const int32_t* tok, float2* part,
                  float* ztok, uint32_t* status, cudaStream_t s, int tok_base = 0);
@@ -47,9 +47,12 @@ int bwd_chunk_bf16(int64_t rc, int d, int V, const void* Hpk, const void* W, con
 int bwd_grads_bf16(int64_t rc, int d, int V, const void* Hpk, const void* W, float* dH, float* dW, int dw_accumulate,
                    const void* dz, int64_t ldz, uint32_t* status, cudaStream_t s, int dh_accumulate);
 // The logit store of the forward turned into dZ in place (f16 e -> bf16 dZ), rows [0, N) of already
-// offset pointers; scale [c][lds] (lds: the store's row count, the pitch of its slice maxima).
+// offset pointers; scale [c][lds] (lds: the store's row count, the pitch of its slice maxima). With
+// tok_base, the store holds vocabulary columns [tok_base, tok_base + V) and the one-hot term applies
+// where tok - tok_base is in [0, V).
 int dz_from_store_bf16(int64_t N, int V, void* store, int64_t ldz, const float* scale, int64_t lds,
-                       const int32_t* tok, const float* lse, const float* logp, const float* coef, cudaStream_t s);
+                       const int32_t* tok, const float* lse, const float* logp, const float* coef, cudaStream_t s,
+                       int tok_base = 0);
 int bwd_chunk_f32(int64_t rc, int d, int V, const float* Hpk, const float* W, const int32_t* tok,
                   const float* lse, const float* coef, float* dH, float* dW, int dw_accumulate, float* dz,
                   int64_t ldz, uint32_t* status, cudaStream_t s, int tok_base = 0, int dh_accumulate = 0);

@@ -100,13 +100,14 @@ struct FwdLseStoreEpi {
     float* ztok;
     float* scale;   // [ceil(N / 32)][lds]
     int64_t lds;
+    int tok_base;   // token ids are global; W holds vocabulary rows [tok_base, tok_base + N)
   };
   using State = FwdLseEpi::State;
   static __device__ __forceinline__ int cols(const Params& p) { return p.N; }
   static __device__ __forceinline__ void begin_unit(const Params& p, State& st, int row, int) {
     st.m2 = -INFINITY;
     st.s = 0.f;
-    st.tok = row < p.M ? __ldg(p.tok + row) : -1;
+    st.tok = row < p.M ? __ldg(p.tok + row) - p.tok_base : -1;
   }
   static __device__ __forceinline__ void chunk_to_smem(const Params& p, State& st, int row, int col0,
                                                        const uint32_t (&r)[32], uint8_t* buf, int lane) {
@@ -412,8 +413,9 @@ constexpr int kDzThreads = 256;
 
 __global__ void __launch_bounds__(kDzThreads) dz_from_store_kernel(int64_t N, int V, uint16_t* z, int64_t ldz,
                                                                    const float* scale, int64_t lds,
-                                                                   const int32_t* tok, const float* lse,
-                                                                   const float* logp, const float* coef) {
+                                                                   const int32_t* tok, int tok_base,
+                                                                   const float* lse, const float* logp,
+                                                                   const float* coef) {
   __shared__ float f_s[kDzCols / 32][kDzRows];   // -coef 2^(m - lse log2 e) per slice and row
   __shared__ float one_s[kDzRows];               // coef (1 - p_o)
   __shared__ int tok_s[kDzRows];
@@ -433,7 +435,7 @@ __global__ void __launch_bounds__(kDzThreads) dz_from_store_kernel(int64_t N, in
   }
   if (t < kDzRows) {
     const int64_t row = r0 + t;
-    tok_s[t] = row < N ? __ldg(tok + row) : -1;
+    tok_s[t] = row < N ? __ldg(tok + row) - tok_base : -1;   // outside [0, V): no one-hot term here
     one_s[t] = row < N ? -__ldg(coef + row) * expm1f(__ldg(logp + row)) : 0.f;
   }
   __syncthreads();
@@ -677,12 +679,12 @@ int fwd_gemm_bf16(int64_t N, int d, int V, const void* Hpk, const void* W, const
 // L2 share of hidden rows.
 int fwd_gemm_store_bf16(int64_t N, int d, int V, const void* Hpk, const void* W, const int32_t* tok, float2* part,
                         float* ztok, int splits, void* store, int64_t ldz, float* scale, uint32_t* status,
-                        cudaStream_t s) {
+                        cudaStream_t s, int tok_base) {
   CUtensorMap ta, tb, tc;
   if (!map_kmajor(&ta, Hpk, N, d, d, kBM) || !map_kmajor(&tb, W, V, d, d, kBRowsBox)) return PS_ERR_INVALID_ARG;
   if (!make_map(&tc, store, V, N, ldz * 2, 32, 32, CU_TENSOR_MAP_SWIZZLE_64B, CU_TENSOR_MAP_DATA_TYPE_FLOAT16))
     return PS_ERR_INVALID_ARG;
-  FwdLseStoreEpi::Params ep{tok, static_cast<int>(N), V, part, ztok, scale, N};
+  FwdLseStoreEpi::Params ep{tok, static_cast<int>(N), V, part, ztok, scale, N, tok_base};
   const int workers = num_sms_current();
   int band = static_cast<int>(kFwdBandL2Bytes / (static_cast<double>(kBM) * d * 2.0));
   if (band < 1) band = 1;
@@ -769,11 +771,12 @@ int bwd_grads_bf16(int64_t rc, int d, int V, const void* Hpk, const void* W, flo
 }
 
 int dz_from_store_bf16(int64_t N, int V, void* store, int64_t ldz, const float* scale, int64_t lds,
-                       const int32_t* tok, const float* lse, const float* logp, const float* coef, cudaStream_t s) {
+                       const int32_t* tok, const float* lse, const float* logp, const float* coef, cudaStream_t s,
+                       int tok_base) {
   if (N == 0) return PS_OK;
   const dim3 grid(static_cast<unsigned>((N + kDzRows - 1) / kDzRows), static_cast<unsigned>((V + kDzCols - 1) / kDzCols));
-  dz_from_store_kernel<<<grid, kDzThreads, 0, s>>>(N, V, static_cast<uint16_t*>(store), ldz, scale, lds, tok, lse,
-                                                   logp, coef);
+  dz_from_store_kernel<<<grid, kDzThreads, 0, s>>>(N, V, static_cast<uint16_t*>(store), ldz, scale, lds, tok,
+                                                   tok_base, lse, logp, coef);
   return cudaGetLastError() == cudaSuccess ? PS_OK : PS_ERR_CUDA;
 }
 

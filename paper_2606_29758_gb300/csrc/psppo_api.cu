@@ -663,19 +663,38 @@ static int lmhead_fwd_impl(int64_t N, int d, int V, int dtype, const void* Hpk, 
   return cudaGetLastError() == cudaSuccess ? PS_OK : PS_ERR_CUDA;
 }
 
-// The backward from the logit store: the conversion into dZ (HBM-bound), then dH and dW over all rows.
-// Running the conversion of later rows on a second stream under the dH GEMM of earlier rows (the
-// GEMM's one CTA per SM leaves room for conversion blocks) measured 1-2% slower at the 7B workload
-// (backward 272.7 / 273.0 against 267.3 / 269.2 ms, back to back), so the parts run in turn.
-static int bwd_from_store_run(int64_t N, int d, int V, const void* Hpk, const void* W, const int32_t* tok,
-                              const float* lse, const float* logp, const float* coef, void* store, float* dH,
-                              float* dW, int flags, uint32_t* status, cudaStream_t s) {
+// The backward from a logit store of V vocabulary columns whose first is global token id tok_base.
+static int bwd_from_store_impl(int64_t N, int d, int V, int64_t tok_base, int dtype, const void* Hpk, const void* W,
+                               const int32_t* tok, const float* lse, const float* logp, const float* coef,
+                               void* store, size_t store_bytes, float* dH, float* dW, int flags, void* ws,
+                               size_t ws_bytes, ps_stream_t stream) {
+  if (N < 0 || N > INT32_MAX || V < 1 || !dtype_ok(dtype) || !d_ok(d, dtype)) return PS_ERR_INVALID_ARG;
+  if (flags & ~(PS_DW_ACCUMULATE | PS_DH_ACCUMULATE)) return PS_ERR_INVALID_ARG;
+  if (dtype != PS_DTYPE_BF16) return PS_ERR_UNSUPPORTED;
+  if (N > 0 && (!Hpk || !W || !tok || !lse || !logp || !coef || !store)) return PS_ERR_INVALID_ARG;
+  if ((N > 0 && (!al16(Hpk) || !al16(W) || !al16(store))) || (dH && !al16(dH)) || (dW && !al16(dW)))
+    return PS_ERR_INVALID_ARG;
+  if (N > 0 && store_bytes < store_layout(N, V).bytes) return PS_ERR_WORKSPACE;
+  if (!device_is_sm103()) return PS_ERR_UNSUPPORTED;
+  cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
+  int rc = begin_call(ws, ws_bytes, kWsHeader, s);
+  if (rc != PS_OK) return rc;
+  if (N == 0) {
+    if (dW && !(flags & PS_DW_ACCUMULATE))
+      return cudaMemsetAsync(dW, 0, sizeof(float) * static_cast<size_t>(V) * d, s) == cudaSuccess ? PS_OK
+                                                                                                : PS_ERR_CUDA;
+    return PS_OK;
+  }
+  // the conversion into dZ (HBM-bound), then dH and dW over all rows. Running the conversion of later
+  // rows on a second stream under the dH GEMM of earlier rows (the GEMM's one CTA per SM leaves room
+  // for conversion blocks) measured 1-2% slower at the 7B workload (backward 272.7 / 273.0 against
+  // 267.3 / 269.2 ms, back to back), so the parts run in turn.
   const StoreLayout L = store_layout(N, V);
   const float* scale = reinterpret_cast<const float*>(static_cast<const uint8_t*>(store) + L.scale_off);
-  int rc = dz_from_store_bf16(N, V, store, L.ldz, scale, N, tok, lse, logp, coef, s);
+  rc = dz_from_store_bf16(N, V, store, L.ldz, scale, N, tok, lse, logp, coef, s, static_cast<int>(tok_base));
   if (rc != PS_OK) return rc;
-  return bwd_grads_bf16(N, d, V, Hpk, W, dH, dW, (flags & PS_DW_ACCUMULATE) ? 1 : 0, store, L.ldz, status, s,
-                        (flags & PS_DH_ACCUMULATE) ? 1 : 0);
+  return bwd_grads_bf16(N, d, V, Hpk, W, dH, dW, (flags & PS_DW_ACCUMULATE) ? 1 : 0, store, L.ldz, status_word(ws),
+                        s, (flags & PS_DH_ACCUMULATE) ? 1 : 0);
 }
 
 extern "C" {
@@ -711,38 +730,39 @@ int ps_lmhead_ppo_bwd_from_store(int64_t N, int d, int V, int dtype, const void*
                                  void* store, size_t store_bytes, float* dH, float* dW, int flags, void* ws,
                                  size_t ws_bytes, ps_stream_t stream) {
   NvtxRange nvtx_range("ps_lmhead_ppo_bwd_from_store");
-  if (N < 0 || N > INT32_MAX || V < 1 || !dtype_ok(dtype) || !d_ok(d, dtype)) return PS_ERR_INVALID_ARG;
-  if (flags & ~(PS_DW_ACCUMULATE | PS_DH_ACCUMULATE)) return PS_ERR_INVALID_ARG;
-  if (dtype != PS_DTYPE_BF16) return PS_ERR_UNSUPPORTED;
-  if (N > 0 && (!Hpk || !W || !tok || !lse || !logp || !coef || !store)) return PS_ERR_INVALID_ARG;
-  if ((N > 0 && (!al16(Hpk) || !al16(W) || !al16(store))) || (dH && !al16(dH)) || (dW && !al16(dW)))
-    return PS_ERR_INVALID_ARG;
-  if (N > 0 && store_bytes < store_layout(N, V).bytes) return PS_ERR_WORKSPACE;
-  if (!device_is_sm103()) return PS_ERR_UNSUPPORTED;
-  cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
-  int rc = begin_call(ws, ws_bytes, kWsHeader, s);
-  if (rc != PS_OK) return rc;
-  if (N == 0) {
-    if (dW && !(flags & PS_DW_ACCUMULATE))
-      return cudaMemsetAsync(dW, 0, sizeof(float) * static_cast<size_t>(V) * d, s) == cudaSuccess ? PS_OK
-                                                                                                : PS_ERR_CUDA;
-    return PS_OK;
-  }
-  return bwd_from_store_run(N, d, V, Hpk, W, tok, lse, logp, coef, store, dH, dW, flags, status_word(ws), s);
+  return bwd_from_store_impl(N, d, V, 0, dtype, Hpk, W, tok, lse, logp, coef, store, store_bytes, dH, dW, flags, ws,
+                             ws_bytes, stream);
+}
+
+int ps_lmhead_ppo_bwd_vocab_shard_from_store(int64_t N, int d, int Vs, int64_t v0, int V, int dtype, const void* Hpk,
+                                             const void* W_shard, const int32_t* tok, const float* lse,
+                                             const float* logp, const float* coef, void* store, size_t store_bytes,
+                                             float* dH, float* dW_shard, int flags, void* ws, size_t ws_bytes,
+                                             ps_stream_t stream) {
+  NvtxRange nvtx_range("ps_lmhead_ppo_bwd_vocab_shard_from_store");
+  if (Vs < 1 || v0 < 0 || V < 1 || v0 + Vs > V) return PS_ERR_INVALID_ARG;
+  return bwd_from_store_impl(N, d, Vs, v0, dtype, Hpk, W_shard, tok, lse, logp, coef, store, store_bytes, dH,
+                             dW_shard, flags, ws, ws_bytes, stream);
 }
 
 size_t ps_lmhead_logit_stats_workspace_size(int64_t N, int d, int Vs, int dtype) {
   return ps_lmhead_ppo_fwd_workspace_size(N, d, Vs, dtype);
 }
 
-int ps_lmhead_logit_stats(int64_t N, int d, int Vs, int64_t v0, int dtype, const void* Hpk, const void* W_shard,
-                          const int32_t* tok, float* stats, float* ztok, void* ws, size_t ws_bytes,
-                          ps_stream_t stream) {
-  NvtxRange nvtx_range("ps_lmhead_logit_stats");
+}  // extern "C"
+
+static int logit_stats_impl(int64_t N, int d, int Vs, int64_t v0, int dtype, const void* Hpk, const void* W_shard,
+                            const int32_t* tok, float* stats, float* ztok, void* store, size_t store_bytes, void* ws,
+                            size_t ws_bytes, ps_stream_t stream) {
   if (N < 0 || N > INT32_MAX || Vs < 1 || v0 < 0 || v0 + Vs > INT32_MAX || !dtype_ok(dtype) || !d_ok(d, dtype))
     return PS_ERR_INVALID_ARG;
   if (N > 0 && (!Hpk || !W_shard || !tok || !stats || !ztok)) return PS_ERR_INVALID_ARG;
   if (N > 0 && (!al16(Hpk) || !al16(W_shard) || (reinterpret_cast<uintptr_t>(stats) & 7))) return PS_ERR_INVALID_ARG;
+  if (store != nullptr) {
+    if (dtype != PS_DTYPE_BF16) return PS_ERR_UNSUPPORTED;
+    if (!al16(store)) return PS_ERR_INVALID_ARG;
+    if (store_bytes < store_layout(N, Vs).bytes) return PS_ERR_WORKSPACE;
+  }
   if (dtype == PS_DTYPE_BF16 && !device_is_sm103()) return PS_ERR_UNSUPPORTED;
   cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
   FwdWs f = fwd_ws(ws, N, Vs, dtype, ws_bytes);
@@ -752,7 +772,15 @@ int ps_lmhead_logit_stats(int64_t N, int d, int Vs, int64_t v0, int dtype, const
   int splits;
   if (dtype == PS_DTYPE_BF16) {
     splits = choose_fwd_splits_bf16(N, d, Vs, num_sms_current(), f.splits);
-    rc = fwd_gemm_bf16(N, d, Vs, Hpk, W_shard, tok, f.part, f.ztok, splits, status_word(ws), s, static_cast<int>(v0));
+    if (store) {
+      const StoreLayout L = store_layout(N, Vs);
+      float* scale = reinterpret_cast<float*>(static_cast<uint8_t*>(store) + L.scale_off);
+      rc = fwd_gemm_store_bf16(N, d, Vs, Hpk, W_shard, tok, f.part, f.ztok, splits, store, L.ldz, scale,
+                               status_word(ws), s, static_cast<int>(v0));
+    } else {
+      rc = fwd_gemm_bf16(N, d, Vs, Hpk, W_shard, tok, f.part, f.ztok, splits, status_word(ws), s,
+                         static_cast<int>(v0));
+    }
   } else {
     splits = fwd_splits_f32(Vs);
     rc = fwd_gemm_f32(N, d, Vs, static_cast<const float*>(Hpk), static_cast<const float*>(W_shard), tok, f.part,
@@ -763,6 +791,24 @@ int ps_lmhead_logit_stats(int64_t N, int d, int Vs, int64_t v0, int dtype, const
   stats_merge_kernel<<<static_cast<unsigned>(nb), kFinThreads, 0, s>>>(N, splits, f.part, f.ztok, tok, v0, Vs,
                                                                         reinterpret_cast<float2*>(stats), ztok);
   return cudaGetLastError() == cudaSuccess ? PS_OK : PS_ERR_CUDA;
+}
+
+extern "C" {
+
+int ps_lmhead_logit_stats(int64_t N, int d, int Vs, int64_t v0, int dtype, const void* Hpk, const void* W_shard,
+                          const int32_t* tok, float* stats, float* ztok, void* ws, size_t ws_bytes,
+                          ps_stream_t stream) {
+  NvtxRange nvtx_range("ps_lmhead_logit_stats");
+  return logit_stats_impl(N, d, Vs, v0, dtype, Hpk, W_shard, tok, stats, ztok, nullptr, 0, ws, ws_bytes, stream);
+}
+
+int ps_lmhead_logit_stats_store(int64_t N, int d, int Vs, int64_t v0, int dtype, const void* Hpk,
+                                const void* W_shard, const int32_t* tok, float* stats, float* ztok, void* store,
+                                size_t store_bytes, void* ws, size_t ws_bytes, ps_stream_t stream) {
+  NvtxRange nvtx_range("ps_lmhead_logit_stats_store");
+  if (store == nullptr) return PS_ERR_INVALID_ARG;
+  return logit_stats_impl(N, d, Vs, v0, dtype, Hpk, W_shard, tok, stats, ztok, store, store_bytes, ws, ws_bytes,
+                          stream);
 }
 
 size_t ps_lmhead_ppo_fwd_from_stats_workspace_size(int64_t N) {

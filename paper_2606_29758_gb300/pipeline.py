@@ -225,12 +225,19 @@ class VocabParallelHead:
     12 bytes per row over `group`; nothing with one process, which then holds every shard), the
     identical `forward(...)` on every process, `backward(r, ...)` for every local shard (its dW rows and
     its term of dH, added into dH by every local shard after the first: PS_DH_ACCUMULATE), and
-    `reduce_dH()` (the all_reduce of dH over the processes; nothing with one process)."""
+    `reduce_dH()` (the all_reduce of dH over the processes; nothing with one process).
+
+    With `store`, each shard's statistics call also keeps the shard's logits in a logit store of its
+    own (allocated for the shards this process runs, on their first use) and its backward turns them
+    into the shard's dZ instead of recomputing them (bf16 heads)."""
 
     def __init__(self, shards, capacity: int, d: int, V: int, dtype: torch.dtype = torch.bfloat16,
                  device: str = "cuda", eps: float = 0.2, loss_scale: float = 1.0, bwd_chunk_rows: int = 32768,
-                 group=None):
+                 group=None, store: bool = False):
+        if store and dtype != torch.bfloat16:
+            raise ValueError("the logit store needs a bf16 head")
         self.shards, self.d, self.V, self.eps, self.loss_scale, self.group = list(shards), d, V, eps, loss_scale, group
+        self.device, self.use_store, self.stores = device, store, {}
         self.S = len(self.shards)
         self.dcode = B.dtype_code(torch.empty(0, dtype=dtype))
         f32 = dict(dtype=torch.float32, device=device)
@@ -244,13 +251,21 @@ class VocabParallelHead:
         self.chunk_rows = min(bwd_chunk_rows, capacity)
         self.ws_bwd = torch.zeros(B.ps_lmhead_ppo_bwd_workspace_size(capacity, d, vmax, self.dcode, self.chunk_rows),
                                   **u8)
+        self.ws_store = torch.zeros(B.ps_lmhead_ppo_bwd_from_store_workspace_size(), **u8)
         self.lse, self.logp, self.ratio, self.coef, self.row_loss = (torch.empty(capacity, **f32) for _ in range(5))
         self.loss = torch.zeros(1, dtype=torch.float64, device=device)
 
     def stats(self, r: int, N: int, hid, W_shard, tok):
         v0, Vs = self.shards[r]
-        B.ps_lmhead_logit_stats(N, self.d, Vs, v0, self.dcode, hid, W_shard, tok, self.stats_all[r], self.ztok_all[r],
-                                self.ws_stats)
+        if self.use_store:
+            if r not in self.stores:
+                self.stores[r] = torch.empty(B.ps_lmhead_logit_store_size(self.capacity, Vs), dtype=torch.uint8,
+                                             device=self.device)
+            B.ps_lmhead_logit_stats_store(N, self.d, Vs, v0, self.dcode, hid, W_shard, tok, self.stats_all[r],
+                                          self.ztok_all[r], self.stores[r], self.ws_stats)
+        else:
+            B.ps_lmhead_logit_stats(N, self.d, Vs, v0, self.dcode, hid, W_shard, tok, self.stats_all[r],
+                                    self.ztok_all[r], self.ws_stats)
 
     def gather(self, N: int, rank: int):
         """Every shard's statistics on every process (rank = the index of this process's shard)."""
@@ -272,12 +287,18 @@ class VocabParallelHead:
     def backward(self, r: int, N: int, hid, W_shard, tok, dH, dW_shard, add_to_dH: bool = False):
         """Shard r's rows of dW (overwritten) and its term of dH (written, or added to dH)."""
         v0, Vs = self.shards[r]
+        flags = B.PS_DH_ACCUMULATE if add_to_dH else 0
+        if self.use_store:
+            # the store of this shard's last statistics call becomes its dZ: one backward per call
+            B.ps_lmhead_ppo_bwd_vocab_shard_from_store(N, self.d, Vs, v0, self.V, self.dcode, hid, W_shard, tok,
+                                                       self.lse, self.logp, self.coef, self.stores[r], dH, dW_shard,
+                                                       flags, self.ws_store)
+            return
         # the workspace of chunk_rows rows at this shard's width: every shard (and the whole head with
         # the same chunk_rows) cuts the rows into the same chunks
         nb = B.ps_lmhead_ppo_bwd_workspace_size(self.capacity, self.d, Vs, self.dcode, self.chunk_rows)
         B.ps_lmhead_ppo_bwd_vocab_shard(N, self.d, Vs, v0, self.V, self.dcode, hid, W_shard, tok, self.lse,
-                                        self.coef, dH, dW_shard, B.PS_DH_ACCUMULATE if add_to_dH else 0,
-                                        self.ws_bwd[:nb])
+                                        self.coef, dH, dW_shard, flags, self.ws_bwd[:nb])
 
     def reduce_dH(self, dH):
         import torch.distributed as dist

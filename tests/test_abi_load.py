@@ -158,3 +158,22 @@ def test_logit_store_layout_and_refusals_on_the_host(lib):
     assert bwd(0, None, need) == INV
     assert bwd(0, fake, need, flags=4) == INV                     # unknown flag
     assert bwd(0, fake, need - 1) == WS
+
+
+def test_vocabulary_shard_store_refusals_on_the_host(lib):
+    import ctypes
+    L = lib
+    INV, UNSUP, WS = 1, 2, 3
+    fake = ctypes.c_void_p(1 << 20)
+    need = L.ps_lmhead_logit_store_size(10, 64)
+    stats = lambda dt, store, nbytes, v0=0: L.ps_lmhead_logit_stats_store(  # noqa: E731
+        10, 128, 64, v0, dt, fake, fake, fake, fake, fake, store, nbytes, None, 0, None)
+    assert stats(0, None, need) == INV
+    assert stats(1, fake, need) == UNSUP
+    assert stats(0, fake, need - 1) == WS
+    assert stats(0, fake, need, v0=-1) == INV
+    bwd = lambda Vs, v0, V, dt=0, nbytes=need: L.ps_lmhead_ppo_bwd_vocab_shard_from_store(  # noqa: E731
+        10, 128, Vs, v0, V, dt, fake, fake, fake, fake, fake, fake, fake, nbytes, fake, fake, 0, None, 0, None)
+    assert bwd(64, 1000, 1024) == INV           # the shard runs past the vocabulary
+    assert bwd(64, 0, 1024, dt=1) == UNSUP
+    assert bwd(64, 0, 1024, nbytes=need - 1) == WS

@@ -10,7 +10,8 @@ and every per-row output (lse, logp, ratio, coef, row loss, dH) bit for bit; the
 sum) to 1e-12 relative; dW within the rounding of a different f32 accumulation order.
 
 The dW bound: dW[v, c] sums the terms dZ_iv h_ic. The shards cut the rows into different 16-row
-MMA steps and backward chunks, so the two results accumulate the same terms in another order.
+MMA steps and backward chunks (or, from the logit store, one launch over each pass's rows), so the
+two results accumulate the same terms in another order.
 Every accumulation step (a 16-deep MMA into the f32 accumulator in TMEM, or the addition of a
 chunk's partial to dW) errs by at most 2 ulps (2^-22 relative) of a partial sum whose magnitude
 is at most S[v, c] = sum_i |dZ_iv| |h_ic|. So |dW_shards - dW_whole| <= 2 n_acc 2^-22 S per entry,
@@ -43,8 +44,11 @@ ROW_OUTS = ("src_row", "row_traj", "row_pos", "tok", "oldlogp", "w", "adv", "lse
             "row_loss")
 
 
-@pytest.mark.parametrize("name,world", [("mid", 2), ("1.5b", 2), ("1.5b", 3)])
-def test_prompt_shards_reproduce_the_whole_batch(name, world):
+@pytest.mark.parametrize("name,world,store", [("mid", 2, False), ("1.5b", 2, False), ("1.5b", 3, False),
+                                              ("mid", 2, True), ("1.5b", 3, True)])
+def test_prompt_shards_reproduce_the_whole_batch(name, world, store):
+    # store: the logits kept in the logit store by every pass (whole batch and shards); the shards'
+    # backward converts each shard's store and accumulates dW over all of its rows in one launch
     from paper_2606_29758_gb300 import PS_MODE_TRUNC, PassShape, UpdatePass, prompt_shard
     from paper_2606_29758_gb300 import _binding as B
     cfg = get_config(name)
@@ -52,7 +56,8 @@ def test_prompt_shards_reproduce_the_whole_batch(name, world):
     D = b.dev
     chunk = 65536 if cfg.V > 100000 else 256
     dt = torch.bfloat16
-    whole = UpdatePass(PassShape(cfg.P, cfg.K, b.T_max, cfg.d, cfg.V, b.total_len, dt, chunk), eps=cfg.eps,
+    whole = UpdatePass(PassShape(cfg.P, cfg.K, b.T_max, cfg.d, cfg.V, b.total_len, dt, chunk,
+                                 b.total_len if store else 0), eps=cfg.eps,
                        loss_scale=cfg.loss_scale, mode=PS_MODE_TRUNC)
     N = whole.run(D["q"], D["L"], D["R"], D["tok_full"], D["oldlogp_full"], D["hid_full"], D["W"], cfg.seed, cfg.step)
     torch.cuda.synchronize()
@@ -64,14 +69,21 @@ def test_prompt_shards_reproduce_the_whole_batch(name, world):
     chunks = [r1 - r0 for r0, r1 in bwd_chunks(N, chunk)]
     for rank in range(world):
         sh = prompt_shard(cfg.P, cfg.K, b.L, world, rank)
-        up = UpdatePass(PassShape(sh.prompts, cfg.K, b.T_max, cfg.d, cfg.V, sh.o1 - sh.o0, dt, chunk), eps=cfg.eps,
+        up = UpdatePass(PassShape(sh.prompts, cfg.K, b.T_max, cfg.d, cfg.V, sh.o1 - sh.o0, dt, chunk,
+                                  sh.o1 - sh.o0 if store else 0), eps=cfg.eps,
                         loss_scale=cfg.loss_scale, mode=PS_MODE_TRUNC)     # the global scale 1/(P K)
         up.sample(D["q"][sh.p0:sh.p1], D["L"][sh.k0:sh.k1], cfg.seed, cfg.step, traj_base=sh.k0)
         n = up.pack(D["L"][sh.k0:sh.k1], D["R"][sh.k0:sh.k1], D["tok_full"][sh.o0:sh.o1],
                     D["oldlogp_full"][sh.o0:sh.o1], D["hid_full"][sh.o0:sh.o1])
         up.forward(D["W"])
-        B.ps_lmhead_ppo_bwd(n, cfg.d, cfg.V, up.dcode, up.hid, D["W"], up.tok, up.lse, up.coef, up.dH, dW,
-                            B.PS_DW_ACCUMULATE if rank > 0 else B.PS_DW_OVERWRITE, up.ws_bwd)
+        flags = B.PS_DW_ACCUMULATE if rank > 0 else B.PS_DW_OVERWRITE
+        if store:
+            assert up.stored and whole.stored is False      # the whole pass's backward has consumed its store
+            B.ps_lmhead_ppo_bwd_from_store(n, cfg.d, cfg.V, up.dcode, up.hid, D["W"], up.tok, up.lse, up.logp,
+                                           up.coef, up.store, up.dH, dW, flags, up.ws_bwd)
+        else:
+            B.ps_lmhead_ppo_bwd(n, cfg.d, cfg.V, up.dcode, up.hid, D["W"], up.tok, up.lse, up.coef, up.dH, dW,
+                                flags, up.ws_bwd)
         torch.cuda.synchronize()
         up.check_status()
         # cutoffs, weights and packing: the whole batch's, shifted to the shard
@@ -92,12 +104,13 @@ def test_prompt_shards_reproduce_the_whole_batch(name, world):
     assert row0 == N
     loss_rel = abs(loss - whole.loss.item()) / abs(whole.loss.item())
     diff = (dW - whole.dW).abs()
-    n_acc = -(-max(chunks) // 16) + len(chunks)
+    # the store path's dW runs over all of a pass's rows in one launch, accumulated over the shards
+    n_acc = -(-N // 16) + world if store else -(-max(chunks) // 16) + len(chunks)
     S = _abs_term_sums(whole.hid[:N], D["W"], whole.tok[:N], whole.lse[:N], whole.coef[:N])
     viol = (diff / (2 * n_acc * 2.0 ** -22 * S + 1e-30)).max().item()
     dw_rel = (diff.max() / whole.dW.abs().max()).item()
     fro = (diff.norm() / whole.dW.norm()).item()
-    print(name, world, "N", N, "loss rel", loss_rel, "dW max-rel", dw_rel, "Frobenius rel", fro,
+    print(name, world, "store" if store else "recompute", "N", N, "loss rel", loss_rel, "dW max-rel", dw_rel, "Frobenius rel", fro,
           "worst entry / bound", viol, "n_acc", n_acc)
     assert loss_rel < 1e-12, loss_rel
     assert torch.isfinite(dW).all() and viol <= 1.0, viol

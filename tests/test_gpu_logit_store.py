@@ -272,3 +272,27 @@ def test_store_at_full_size(name):
     print(name, N, "rows", len(rows), "dH max-rel", err_h, "dZ worst / bound", worst, "dW store vs recompute", err_w)
     assert err_w < 1e-2
     assert torch.isfinite(sto.dW).all() and torch.isfinite(sto.dH[:N]).all()
+
+
+def test_update_pass_recomputes_when_the_store_is_too_small():
+    # a step with more rows than the store holds takes the recompute path (bit-identical to a pass
+    # without a store); one that fits takes the store
+    cfg = get_config("mid")
+    b = make_batch(cfg, device="cuda")
+    D = b.dev
+    rec, _ = _two_passes(cfg, b, store_rows=0)
+    args = (D["q"], D["L"], D["R"], D["tok_full"], D["oldlogp_full"], D["hid_full"], D["W"], cfg.seed, cfg.step)
+    N = rec.run(*args)
+    _, small = _two_passes(cfg, b, store_rows=N - 1)
+    _, fits = _two_passes(cfg, b, store_rows=N)
+    assert small.run(*args, grads=False) == N and not small.stored
+    assert fits.run(*args, grads=False) == N and fits.stored
+    small.backward(D["W"])
+    fits.backward(D["W"])
+    torch.cuda.synchronize()
+    for up in (rec, small, fits):
+        up.check_status()
+    assert torch.equal(small.dH[:N], rec.dH[:N]) and torch.equal(small.dW, rec.dW)
+    assert small.loss.item() == rec.loss.item() == fits.loss.item()
+    assert not torch.equal(fits.dW, rec.dW)          # the store's dZ rounds differently
+    assert maxrel(fits.dW.double().cpu().numpy(), rec.dW.double().cpu().numpy()) < 1e-2

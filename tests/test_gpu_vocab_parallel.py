@@ -149,3 +149,52 @@ def test_vocab_shards_at_the_7b_head_with_several_chunks():
     assert torch.equal(dW, up.dW)
     _check_dh(f"7b_p2 {N}", dH[:N], up.dH[:N], up.hid[:N], W, up.tok[:N], up.lse[:N], up.coef[:N], cfg.V,
               len(shards))
+
+
+@pytest.mark.parametrize("name", ["mid", "head7b_small"])
+def test_vocab_shards_with_logit_stores(name):
+    # every shard keeps its logits in a store of its own (ps_lmhead_logit_stats_store) and its backward
+    # converts it (ps_lmhead_ppo_bwd_vocab_shard_from_store): the statistics equal the plain calls' bit for
+    # bit (the same sums in the same order), and the gradients match the oracle and the shards that
+    # recompute
+    from paper_2606_29758_gb300 import PassShape, UpdatePass, VocabParallelHead
+    cfg = get_config(name)
+    b = make_batch(cfg, device="cuda")
+    D = b.dev
+    up = UpdatePass(PassShape(cfg.P, cfg.K, b.T_max, cfg.d, cfg.V, b.total_len, torch.bfloat16, 256), eps=cfg.eps,
+                    loss_scale=cfg.loss_scale)
+    N = up.run(D["q"], D["L"], D["R"], D["tok_full"], D["oldlogp_full"], D["hid_full"], D["W"], cfg.seed, cfg.step)
+    torch.cuda.synchronize()
+    _, _, _, _, pk = oracle_prefix(cfg, b)
+    W = D["W"]
+    from oracle import lmhead
+    from oracle.pipeline import widen
+    Hs, W64 = widen(cfg, pk["hid"]), widen(cfg, b.W)
+    f = lmhead.forward(Hs, W64, pk["tok"], pk["oldlogp"], pk["adv"], pk["w"], cfg.eps, cfg.loss_scale)
+    dH_ref, dW_ref = lmhead.backward(Hs, W64, pk["tok"], f["lse"], f["coef"])
+    for shards in _shard_layouts(cfg.V):
+        heads = {}
+        for store in (False, True):
+            vp = VocabParallelHead(shards, b.total_len, cfg.d, cfg.V, torch.bfloat16, eps=cfg.eps,
+                                   loss_scale=cfg.loss_scale, bwd_chunk_rows=256, store=store)
+            for r, (v0, Vs) in enumerate(shards):
+                vp.stats(r, N, up.hid, W[v0:v0 + Vs], up.tok)
+            vp.forward(N, up.tok, up.oldlogp, up.adv, up.w)
+            dH = torch.full_like(up.dH, float("nan"))
+            dW = torch.full_like(up.dW, float("nan"))
+            for r, (v0, Vs) in enumerate(shards):
+                vp.backward(r, N, up.hid, W[v0:v0 + Vs], up.tok, dH, dW[v0:v0 + Vs], add_to_dH=r > 0)
+            torch.cuda.synchronize()
+            heads[store] = (vp, dH, dW)
+        plain, stored = heads[False][0], heads[True][0]
+        assert torch.equal(stored.stats_all[:, :N], plain.stats_all[:, :N])
+        assert torch.equal(stored.ztok_all[:, :N], plain.ztok_all[:, :N])
+        assert stored.loss.item() == plain.loss.item()
+        _, dH_s, dW_s = heads[True]
+        _, dH_p, dW_p = heads[False]
+        e_h = maxrel(dH_s[:N].double().cpu().numpy(), dH_ref)
+        e_w = maxrel(dW_s.double().cpu().numpy(), dW_ref)
+        print(name, shards, "store: dH", e_h, "dW", e_w, "vs recomputing shards: dW",
+              maxrel(dW_s.double().cpu().numpy(), dW_p.double().cpu().numpy()))
+        assert torch.isfinite(dH_s[:N]).all() and torch.isfinite(dW_s).all()
+        assert e_h < GRAD_MAXREL and e_w < GRAD_MAXREL
