@@ -381,8 +381,10 @@ def run_ours(args):
     def vocab_parallel_run(S):
         from paper_2606_29758_gb300 import VocabParallelHead, vocab_shards
         shards = vocab_shards(cfg.V, S)
+        # the shards keep their logits when the whole-head step does (stores of their own, beside the
+        # whole head's)
         vp = VocabParallelHead(shards, b.total_len, cfg.d, cfg.V, tdtype, device=dev, eps=cfg.eps,
-                               loss_scale=up.loss_scale, bwd_chunk_rows=args.chunk_rows)
+                               loss_scale=up.loss_scale, bwd_chunk_rows=args.chunk_rows, store=store_rows > 0)
         W = D["W"]
 
         def vstep(i):
@@ -407,6 +409,7 @@ def run_ours(args):
         del vp
         return {"shards": S, "ms_per_step": v_ms, "tokens_per_s": v_rows / (v_ms * 3e-3),
                 "step_time_ratio_over_whole_head": v_ms / (ms / args.steps),
+                "logits": "kept in a store per shard" if store_rows > 0 else "recomputed",
                 "note": "the same steps with W split into vocabulary shards run one after another on this device "
                         "(logit statistics per shard, the forward from them, each shard's backward); 3 timed steps"}
 
