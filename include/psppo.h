@@ -159,13 +159,14 @@ int ps_pack_prefixes(int P, int K, int T_max, int d, int dtype,
  * (f32 CUDA cores). tok [N] int32 (0 <= tok < V, else PS_DEV_BAD_TOKEN), oldlogp,
  * adv, w [N] f32. Outputs: loss [1] f64 (device), lse, logp, ratio, coef [N] f32,
  * row_loss [N] f32 (may be NULL). Only O(N) values are written; the N x V logits
- * are never stored.
- * Workspace: ps_lmhead_ppo_fwd_workspace_size() bytes hold one (max, sum) partial per row
- * for every 256-column vocabulary tile (bf16: 8 B x ceil(V/256) per row, plus 4 B per row
- * and a few KB), the fastest schedule. A smaller bf16 workspace is accepted down to one
- * partial per row; the forward then splits the vocabulary into as many ranges as fit
- * (more passes over W). f32 needs the full size. Too small: PS_ERR_WORKSPACE, nothing
- * launched.
+ * are never stored (ps_lmhead_ppo_fwd_store below keeps them).
+ * Workspace: ps_lmhead_ppo_fwd_workspace_size() bytes hold the (max, sum) partials of
+ * every row for every 256-column vocabulary tile, the fastest schedule: bf16 two per tile
+ * (one per half of the tile's columns: 16 B x ceil(V/256) per row), f32 one per 64-column
+ * tile, plus 4 B per row and a few KB. A smaller bf16 workspace is accepted down to one
+ * vocabulary range per row (16 B); the forward then splits the vocabulary into as many
+ * ranges as fit (more passes over W). f32 needs the full size. Too small:
+ * PS_ERR_WORKSPACE, nothing launched.
  * Limits: N >= 0 (N = 0 writes loss = 0), 1 <= V < 2^31, d >= 8 and d % 8 == 0 (bf16)
  * or d % 4 == 0 (f32); 16-byte aligned Hpk and W.
  * ------------------------------------------------------------------------- */
@@ -416,9 +417,9 @@ int ps_design_cutoffs(int P, int K, int T_max, const int32_t* L, const float* ga
  * library routine).
  *  - Memory: every GPU that loads the library holds the 64 MiB array until the
  *    process exits.
- *  - Limit: the forward takes as many vocabulary partials per row as 64 MiB hold. For bf16
- *    it needs at least one (12 bytes per packed row plus a few KB: about 5.5 million rows);
- *    all ceil(V/256) of them, the fastest schedule, fit up to about 14,000 rows at
+ *  - Limit: the forward takes as many vocabulary ranges per row as 64 MiB hold. For bf16
+ *    it needs at least one (20 bytes per packed row plus a few KB: about 3.3 million
+ *    rows); all ceil(V/256) of them, the fastest schedule, fit up to about 7,000 rows at
  *    V = 152064. For f32, N * ceil(V/64) * 8 bytes must fit. Larger problems return
  *    PS_ERR_UNSUPPORTED and launch nothing.
  *  - Set-up: the first call in each device context looks up the array's device

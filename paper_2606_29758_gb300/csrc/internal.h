@@ -9,12 +9,15 @@ namespace psk {
 int num_sms_current();
 int device_is_sm103();
 
-// Forward GEMM with the online-logsumexp epilogue. part: [splits][N] (max2, sum) pairs
-// (max in log2 units); ztok: [N] chosen-token logit, written only for rows whose token id minus
+// Forward GEMM with the online-logsumexp epilogue. part: [splits * fwd_partials_per_split_bf16()][N]
+// (max2, sum) pairs (max in log2 units); ztok: [N] chosen-token logit, written only for rows whose token id minus
 // tok_base falls in [0, V) (W holding vocabulary rows [tok_base, tok_base + V) of a sharded head).
-int fwd_tile_splits_bf16(int V);   // one partial per 256-column vocabulary tile
-// Vocabulary ranges per row block, at most max_splits (the partials the workspace holds); the
-// score proxy uses the same chooser.
+int fwd_tile_splits_bf16(int V);   // one vocabulary range per 256-column vocabulary tile
+// (max, sum) partials per vocabulary range of the bf16 forward (one per column group of its
+// epilogue): part holds [splits * this][N] entries.
+int fwd_partials_per_split_bf16();
+// Vocabulary ranges per row block, at most max_splits (the ranges whose partials the workspace
+// holds); the score proxy uses the same chooser.
 int choose_fwd_splits_bf16(int64_t N, int d, int V, int num_sms, int max_splits);
 int fwd_gemm_bf16(int64_t N, int d, int V, const void* Hpk, const void* W, const int32_t* tok, float2* part,
                   float* ztok, int splits, uint32_t* status, cudaStream_t s, int tok_base = 0);

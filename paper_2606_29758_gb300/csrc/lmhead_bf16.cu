@@ -32,6 +32,7 @@ static __device__ __forceinline__ float pick32(const uint32_t (&r)[32], int j) {
 }
 
 struct FwdLseEpi {
+  static constexpr int kEpiWarps = 8;   // two column groups per row: two (max, sum) partials per unit
   static constexpr bool kTmaStore = false;
   struct Params {
     const int32_t* tok;
@@ -92,6 +93,7 @@ struct FwdLseEpi {
 // scale[slice][row]. The sums use the same e_v, in the same order as FwdLseEpi, so lse is the same.
 // The backward turns e into dZ = coef (1[v = o] - e 2^(m - lse log2 e)) in place.
 struct FwdLseStoreEpi {
+  static constexpr int kEpiWarps = 8;   // as FwdLseEpi
   static constexpr bool kTmaStore = true;
   struct Params {
     const int32_t* tok;
@@ -160,6 +162,7 @@ struct FwdLseStoreEpi {
 // that ||e_o - p||^2 = (r1^2 + r2) / (e_o + r1)^2 keeps its relative accuracy when p(o) -> 1
 // (1 - 2 p(o) + ||p||^2 would cancel there).
 struct FwdProxyEpi {
+  static constexpr int kEpiWarps = 4;
   static constexpr bool kTmaStore = false;
   struct Params {
     const int32_t* tok;
@@ -231,6 +234,7 @@ struct FwdProxyEpi {
 // registers; only the values of a 32-column slice above the current 16th value are inserted.
 constexpr int kTopK = 16;
 struct FwdProxyTopkEpi {
+  static constexpr int kEpiWarps = 4;
   static constexpr bool kTmaStore = false;
   struct Params {
     const int32_t* tok;
@@ -301,6 +305,7 @@ struct FwdProxyTopkEpi {
 // store (coalesced 64-byte row segments; rows beyond the chunk and columns beyond V are clipped by
 // the store itself).
 struct BwdDzEpi {
+  static constexpr int kEpiWarps = 8;   // no per-row state: the two column groups store their own slices
   static constexpr bool kTmaStore = true;
   struct Params {
     const int32_t* tok;
@@ -363,6 +368,7 @@ struct BwdDzEpi {
 };
 
 struct StoreF32Epi {
+  static constexpr int kEpiWarps = 4;   // its K loops are long: the epilogue is a small share
   static constexpr bool kTmaStore = false;
   struct Params {
     float* out;
@@ -536,12 +542,13 @@ static int launch_gemm_single(const CUtensorMap& ta, const CUtensorMap& tb, cons
   if (sc.num_units == 0) return PS_OK;
   if (sc.num_kb == 0) return PS_ERR_INVALID_ARG;
   auto kern = umma_gemm_kernel<A_MN, B_MN, Epi, HALVES>;
-  constexpr size_t smem = gemm_smem_bytes<HALVES>();
+  constexpr int EW = EpiWarps<Epi>::value;
+  constexpr size_t smem = gemm_smem_bytes<HALVES, EW>();
   if (cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, static_cast<int>(smem)) !=
       cudaSuccess)
     return PS_ERR_CUDA;
   const int grid = sc.num_units < num_sms_current() ? sc.num_units : num_sms_current();
-  kern<<<grid, kGemmThreads, smem, s>>>(ta, tb, tc, sc, ep, status, kDefaultTimeoutNs);
+  kern<<<grid, 64 + 32 * EW, smem, s>>>(ta, tb, tc, sc, ep, status, kDefaultTimeoutNs);
   return cudaGetLastError() == cudaSuccess ? PS_OK : PS_ERR_CUDA;
 }
 
@@ -598,6 +605,10 @@ static int launch_gemm(bool pair, const CUtensorMap& ta, const CUtensorMap& tb, 
 }
 
 int fwd_tile_splits_bf16(int V) { return (V + kBN - 1) / kBN; }
+int fwd_partials_per_split_bf16() {
+  static_assert(FwdLseEpi::kEpiWarps == FwdLseStoreEpi::kEpiWarps, "the two forwards write the same partials");
+  return FwdLseEpi::kEpiWarps / 4;
+}
 
 // Pick the number of vocabulary ranges per row block (at most max_splits): the makespan of a
 // static round-robin over `workers`, in tiles, is rounds x tiles per unit. Among the split
@@ -672,24 +683,24 @@ int fwd_gemm_bf16(int64_t N, int d, int V, const void* Hpk, const void* W, const
 }
 
 // The forward that keeps its logits: f16 e [N][ldz] through TMA (32 x 32 boxes from 64-byte-swizzled
-// staging) and the slice maxima scale [ceil(V / 32)][N]. Its epilogue also stages and stores every
-// slice; on 128-row tiles with two TMEM accumulators it overlaps the next tile's MMAs completely,
-// which measured about 1% faster at the 7B workload than the wide tiles of the plain forward
-// (137.2 against 138.7 ms per forward, two back-to-back pairs). The band keeps the plain forward's
-// L2 share of hidden rows.
+// staging) and the slice maxima scale [ceil(V / 32)][N], on the plain forward's tiles and schedule.
+// With 8 epilogue warps the wide tile's epilogue, which also stages and stores every slice, holds
+// each TMEM half for half as long: 131.4 / 131.7 ms per 7B forward against 135.9 / 136.8 ms for 4
+// epilogue warps on 128-row tiles (back to back).
 int fwd_gemm_store_bf16(int64_t N, int d, int V, const void* Hpk, const void* W, const int32_t* tok, float2* part,
                         float* ztok, int splits, void* store, int64_t ldz, float* scale, uint32_t* status,
                         cudaStream_t s, int tok_base) {
+  const int halves = fwd_halves(d);
   CUtensorMap ta, tb, tc;
-  if (!map_kmajor(&ta, Hpk, N, d, d, kBM) || !map_kmajor(&tb, W, V, d, d, kBRowsBox)) return PS_ERR_INVALID_ARG;
+  if (!map_kmajor(&ta, Hpk, N, d, d, kBM * halves) || !map_kmajor(&tb, W, V, d, d, kBRowsBox)) return PS_ERR_INVALID_ARG;
   if (!make_map(&tc, store, V, N, ldz * 2, 32, 32, CU_TENSOR_MAP_SWIZZLE_64B, CU_TENSOR_MAP_DATA_TYPE_FLOAT16))
     return PS_ERR_INVALID_ARG;
   FwdLseStoreEpi::Params ep{tok, static_cast<int>(N), V, part, ztok, scale, N, tok_base};
   const int workers = num_sms_current();
-  int band = static_cast<int>(kFwdBandL2Bytes / (static_cast<double>(kBM) * d * 2.0));
-  if (band < 1) band = 1;
-  if (splits != fwd_tile_splits_bf16(V)) band = (workers + splits - 1) / splits;
-  return launch_gemm_single<false, false, FwdLseStoreEpi, 1>(ta, tb, tc, N, V, d, splits, band, ep, status, s);
+  const int band = splits == fwd_tile_splits_bf16(V) ? fwd_band_max(d) : (workers + splits - 1) / splits;
+  if (halves == 1)
+    return launch_gemm_single<false, false, FwdLseStoreEpi, 1>(ta, tb, tc, N, V, d, splits, band, ep, status, s);
+  return launch_gemm_single<false, false, FwdLseStoreEpi, 2>(ta, tb, tc, N, V, d, splits, band, ep, status, s);
 }
 
 // Bands (row blocks walked together) of the backward GEMMs. Recompute: 32 row blocks of 128 rows

@@ -449,10 +449,10 @@ __global__ void __launch_bounds__(1024) loss_reduce_kernel(int64_t nblocks, cons
 }
 
 // Forward workspace: header | ztok [N] f32 | block_loss [nb] f64 | part [S][N] float2. The
-// (max, sum of exp) partials come last: S, the number of vocabulary ranges per row, is as many
-// as the workspace holds, up to one per 256-column vocabulary tile (bf16) -- at that count every
-// unit of the forward GEMM is one tile, the schedule that keeps W traffic lowest. f32 always
-// uses one partial per 64-column tile.
+// (max, sum of exp) partials come last: S is as many as the workspace holds, up to two per
+// 256-column vocabulary tile (bf16: one per column group of the forward's epilogue, so the
+// vocabulary ranges per row are S / 2; at one range per tile every unit of the forward GEMM is one
+// tile, the schedule that keeps W traffic lowest). f32 always uses one partial per 64-column tile.
 struct FwdWs {
   float2* part;
   float* ztok;
@@ -461,8 +461,10 @@ struct FwdWs {
   size_t bytes;     // bytes used with that S
 };
 static int fwd_full_splits(int V, int dtype) {
-  return dtype == PS_DTYPE_BF16 ? fwd_tile_splits_bf16(V) : fwd_splits_f32(V);
+  return dtype == PS_DTYPE_BF16 ? fwd_tile_splits_bf16(V) * fwd_partials_per_split_bf16() : fwd_splits_f32(V);
 }
+// Partials per vocabulary range, and the fewest partials a forward can run with.
+static int fwd_group(int dtype) { return dtype == PS_DTYPE_BF16 ? fwd_partials_per_split_bf16() : 1; }
 static size_t fwd_fixed_bytes(int64_t N) {
   const int64_t nb = (N + kFinThreads - 1) / kFinThreads;
   return kWsHeader + align_up(sizeof(float) * N, 256) + align_up(sizeof(double) * (nb > 0 ? nb : 1), 256);
@@ -478,15 +480,16 @@ static FwdWs fwd_ws(void* ws, int64_t N, int V, int dtype, size_t ws_bytes) {
   f.ztok = reinterpret_cast<float*>(base + kWsHeader);
   f.block_loss = reinterpret_cast<double*>(base + kWsHeader + align_up(sizeof(float) * N, 256));
   f.part = reinterpret_cast<float2*>(base + fixed);
+  const int g = fwd_group(dtype);
   int S = full;
   if (ws_bytes != SIZE_MAX && N > 0) {
     const size_t room = ws_bytes > fixed ? ws_bytes - fixed : 0;
     const size_t fit = room / (sizeof(float2) * static_cast<size_t>(N));
-    if (fit < static_cast<size_t>(S)) S = static_cast<int>(fit);
+    if (fit < static_cast<size_t>(S)) S = static_cast<int>(fit) / g * g;   // whole vocabulary ranges
     if (dtype != PS_DTYPE_BF16 && S < full) S = 0;   // the f32 kernel needs every partial
   }
   f.splits = S;
-  f.bytes = fixed + fwd_part_bytes(N, S > 0 ? S : 1);
+  f.bytes = fixed + fwd_part_bytes(N, S > 0 ? S : g);
   return f;
 }
 
@@ -640,14 +643,17 @@ static int lmhead_fwd_impl(int64_t N, int d, int V, int dtype, const void* Hpk, 
   if (N == 0) return cudaMemsetAsync(loss, 0, sizeof(double), s) == cudaSuccess ? PS_OK : PS_ERR_CUDA;
   int splits;
   if (dtype == PS_DTYPE_BF16) {
-    splits = choose_fwd_splits_bf16(N, d, V, num_sms_current(), f.splits);
+    const int g = fwd_partials_per_split_bf16();
+    const int ranges = choose_fwd_splits_bf16(N, d, V, num_sms_current(), f.splits / g);
     if (store) {
       const StoreLayout L = store_layout(N, V);
       float* scale = reinterpret_cast<float*>(static_cast<uint8_t*>(store) + L.scale_off);
-      rc = fwd_gemm_store_bf16(N, d, V, Hpk, W, tok, f.part, f.ztok, splits, store, L.ldz, scale, status_word(ws), s);
+      rc = fwd_gemm_store_bf16(N, d, V, Hpk, W, tok, f.part, f.ztok, ranges, store, L.ldz, scale, status_word(ws),
+                               s);
     } else {
-      rc = fwd_gemm_bf16(N, d, V, Hpk, W, tok, f.part, f.ztok, splits, status_word(ws), s);
+      rc = fwd_gemm_bf16(N, d, V, Hpk, W, tok, f.part, f.ztok, ranges, status_word(ws), s);
     }
+    splits = ranges * g;   // the partials the finalize merges
   } else {
     splits = fwd_splits_f32(V);
     rc = fwd_gemm_f32(N, d, V, static_cast<const float*>(Hpk), static_cast<const float*>(W), tok, f.part, f.ztok,
@@ -771,16 +777,18 @@ static int logit_stats_impl(int64_t N, int d, int Vs, int64_t v0, int dtype, con
   if (rc != PS_OK || N == 0) return rc;
   int splits;
   if (dtype == PS_DTYPE_BF16) {
-    splits = choose_fwd_splits_bf16(N, d, Vs, num_sms_current(), f.splits);
+    const int g = fwd_partials_per_split_bf16();
+    const int ranges = choose_fwd_splits_bf16(N, d, Vs, num_sms_current(), f.splits / g);
     if (store) {
       const StoreLayout L = store_layout(N, Vs);
       float* scale = reinterpret_cast<float*>(static_cast<uint8_t*>(store) + L.scale_off);
-      rc = fwd_gemm_store_bf16(N, d, Vs, Hpk, W_shard, tok, f.part, f.ztok, splits, store, L.ldz, scale,
+      rc = fwd_gemm_store_bf16(N, d, Vs, Hpk, W_shard, tok, f.part, f.ztok, ranges, store, L.ldz, scale,
                                status_word(ws), s, static_cast<int>(v0));
     } else {
-      rc = fwd_gemm_bf16(N, d, Vs, Hpk, W_shard, tok, f.part, f.ztok, splits, status_word(ws), s,
+      rc = fwd_gemm_bf16(N, d, Vs, Hpk, W_shard, tok, f.part, f.ztok, ranges, status_word(ws), s,
                          static_cast<int>(v0));
     }
+    splits = ranges * g;   // the partials the merge reads
   } else {
     splits = fwd_splits_f32(Vs);
     rc = fwd_gemm_f32(N, d, Vs, static_cast<const float*>(Hpk), static_cast<const float*>(W_shard), tok, f.part,

@@ -4,11 +4,12 @@
 //
 // A is K-major ([M][K] in memory) or MN-major ([K][M]); likewise B ([N][K] or [K][N]).
 // Tiles of 128 x 256 or 256 x 256 outputs (HALVES, below), 64-deep K blocks, a shared-memory
-// ring fed by TMA with 128-byte swizzle. Roles (192 threads):
+// ring fed by TMA with 128-byte swizzle. Roles (64 + 32 x Epi::kEpiWarps threads):
 //   warp 0      TMA producer (one lane)
 //   warp 1      TMEM allocator + MMA issuer (one lane)
-//   warps 2..5  epilogue: each thread owns one accumulator row (TMEM lane) and reads
-//               its 256 columns in chunks of 32 with tcgen05.ld
+//   warps 2..   epilogue: each thread owns one accumulator row (TMEM lane) and reads its
+//               256 columns in chunks of 32 with tcgen05.ld; with 8 epilogue warps two warps
+//               share each TMEM lane quarter, one reading columns 0..127 and one 128..255
 // An epilogue either stores from registers itself or (Epi::kTmaStore) stages 32 x 32 slices in
 // shared memory for TMA tensor stores through a third map. Every wait is bounded; on expiry the
 // kernel sets PS_DEV_TIMEOUT, waits (bounded) for its own loads in flight, frees TMEM and returns.
@@ -27,7 +28,7 @@ namespace psk {
 constexpr int kBM = 128;
 constexpr int kBN = 256;
 constexpr int kBK = 64;
-constexpr int kGemmThreads = 192;
+constexpr int kGemmThreads = 192;                 // the CTA-pair kernel: 4 epilogue warps
 constexpr uint32_t kTileABytes = kBM * kBK * 2;   // 16 KB
 constexpr uint32_t kTileBBytes = kBN * kBK * 2;   // 32 KB
 constexpr uint32_t kTmemCols = 512;               // two 256-column f32 accumulators
@@ -68,17 +69,30 @@ struct GemmCfg {
   static constexpr int kAccBufs = HALVES == 1 ? 2 : 1;        // accumulator buffers in TMEM
 };
 
-// Epilogues that store through TMA (Epi::kTmaStore) stage each 32-row x 32-column bf16 slice of a
-// warp in shared memory, two buffers per epilogue warp, 64-byte swizzled (a 64-byte row per TMEM
-// lane, its 16-byte units permuted by row bits 1-2, so a warp's stores hit every bank group).
+// Epilogues that store through TMA (Epi::kTmaStore) stage each 32-row x 32-column 2-byte slice of a
+// warp in shared memory, 64-byte swizzled (a 64-byte row per TMEM lane, its 16-byte units permuted
+// by row bits 1-2, so a warp's stores hit every bank group): two buffers per warp with 4 epilogue
+// warps, one with 8 (whose wide-tile ring leaves room for no more).
 constexpr int kStageBytes = 32 * 64;
 
-template <int HALVES>
+// Epilogue warps per CTA: Epi::kEpiWarps, 4 or 8. With 8, each accumulator row is read by two
+// warps (columns 0..127 and 128..255 of every tile), which halves the time an epilogue holds a
+// TMEM half; an epilogue with per-row state then keeps one state per column group, and its
+// per-unit results (the forward's partials) come in two parts.
+template <class Epi>
+struct EpiWarps {
+  static_assert(Epi::kEpiWarps == 4 || Epi::kEpiWarps == 8, "4 or 8 epilogue warps");
+  static constexpr int value = Epi::kEpiWarps;
+};
+template <int EW>
+struct StageBufs { static constexpr int value = EW == 8 ? 1 : 2; };
+
+template <int HALVES, int EW = 4>
 struct GemmSmemT {
   // 1024-byte aligned tile ring first (128-byte swizzle atoms repeat every 1 KB)
   uint8_t a[GemmCfg<HALVES>::kStagesH][GemmCfg<HALVES>::kABytes];
   uint8_t b[GemmCfg<HALVES>::kStagesH][kTileBBytes];
-  uint8_t stage[4][2][kStageBytes];   // store staging of the four epilogue warps (2 KB-aligned)
+  uint8_t stage[EW][StageBufs<EW>::value][kStageBytes];   // store staging of the epilogue warps
   uint64_t full[GemmCfg<HALVES>::kStagesH];
   uint64_t empty[GemmCfg<HALVES>::kStagesH];
   uint64_t tfull[2];
@@ -87,21 +101,27 @@ struct GemmSmemT {
   uint32_t tmem_base;
   int abort;
 };
-template <int HALVES>
-constexpr size_t gemm_smem_bytes() { return sizeof(GemmSmemT<HALVES>) + 1024; }  // + alignment slack
+template <int HALVES, int EW = 4>
+constexpr size_t gemm_smem_bytes() { return sizeof(GemmSmemT<HALVES, EW>) + 1024; }  // + alignment slack
 
-// tmC: the output map of epilogues that store through TMA (unused by the others).
+// tmC: the output map of epilogues that store through TMA (unused by the others). An epilogue's
+// begin_unit / end_unit see the unit's split index times the column groups (1 with 4 epilogue
+// warps, 2 with 8) plus the thread's column group.
 template <bool A_MN, bool B_MN, class Epi, int HALVES = 1>
-__global__ void __launch_bounds__(kGemmThreads, 1)
+__global__ void __launch_bounds__(64 + 32 * EpiWarps<Epi>::value, 1)
     umma_gemm_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmB,
                      const __grid_constant__ CUtensorMap tmC, const Sched sched, const typename Epi::Params ep,
                      uint32_t* status, uint64_t timeout_ns) {
   using Cfg = GemmCfg<HALVES>;
   constexpr int S = Cfg::kStagesH;
   constexpr int NB = Cfg::kAccBufs;
+  constexpr int EW = EpiWarps<Epi>::value;
+  constexpr int G = EW / 4;                 // column groups per TMEM lane quarter
+  constexpr int CPG = (kBN / 32) / G;       // 32-column chunks per group
+  constexpr int SB = StageBufs<EW>::value;
   extern __shared__ uint8_t smem_raw[];
-  GemmSmemT<HALVES>& sm =
-      *reinterpret_cast<GemmSmemT<HALVES>*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
+  GemmSmemT<HALVES, EW>& sm =
+      *reinterpret_cast<GemmSmemT<HALVES, EW>*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
   const int warp = threadIdx.x >> 5;
   const int lane = threadIdx.x & 31;
 
@@ -112,7 +132,7 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
     }
     for (int a = 0; a < 2; ++a) {
       mbar_init(&sm.tfull[a], 1);
-      mbar_init(&sm.tempty[a], 128);
+      mbar_init(&sm.tempty[a], 32 * EW);
     }
     mbar_init(&sm.drain, 1);
     sm.abort = 0;
@@ -258,6 +278,8 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
   } else {
     // ------------------------------------------------------------------ epilogue
     const int quad = warp & 3;                  // TMEM lanes 32*quad .. 32*quad+31
+    const int ew = warp - 2;                    // epilogue warp
+    const int grp = ew >> 2;                    // column group: chunks [grp * CPG, grp * CPG + CPG)
     const int row_in_tile = quad * 32 + lane;
     typename Epi::State st[HALVES];             // a thread owns row r of each half
     uint32_t tile = 0;
@@ -268,7 +290,7 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
       sched.unit(u, m_blk, split, n0, n1);
       const int row0 = m_blk * Cfg::kRows + row_in_tile;
 #pragma unroll
-      for (int h = 0; h < HALVES; ++h) Epi::begin_unit(ep, st[h], row0 + h * kBM, split);
+      for (int h = 0; h < HALVES; ++h) Epi::begin_unit(ep, st[h], row0 + h * kBM, split * G + grp);
       for (int nb = n0; nb < n1; ++nb, ++tile) {
         const uint32_t acc = tile % NB;
         const uint32_t aph = (tile / NB) & 1u;
@@ -283,11 +305,11 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
           const int row = row0 + h * kBM;
           const uint32_t t_row = tmem_base + (static_cast<uint32_t>(quad * 32) << 16) + acc * kBN + h * kBN;
 #pragma unroll 1
-          for (int c = 0; c < kBN / 32; ++c) {
+          for (int c = grp * CPG; c < grp * CPG + CPG; ++c) {
             uint32_t r[32];
             tmem_ld32(t_row + c * 32, r);
             tmem_ld_wait();
-            if (c == kBN / 32 - 1) {
+            if (c == grp * CPG + CPG - 1) {
               // this half of the accumulator has been read: hand it back to the MMA warp (a wide
               // tile returns its two halves one after the other, tempty[0] and tempty[1])
               tc_fence_before();
@@ -297,8 +319,8 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
             if constexpr (Epi::kTmaStore) {
               // the slice goes to a staging buffer, then one lane stores the warp's 32 x 32 box
               if (col0 < Epi::cols(ep)) {
-                uint8_t* buf = sm.stage[quad][nstore & 1];
-                if (lane == 0) bulk_wait_group_read<1>();   // the store of two slices ago has read it
+                uint8_t* buf = sm.stage[ew][nstore % SB];
+                if (lane == 0) bulk_wait_group_read<SB - 1>();   // the store that last used it has read it
                 __syncwarp();
                 Epi::chunk_to_smem(ep, st[h], row, col0, r, buf, lane);
                 fence_proxy_async_smem();
@@ -317,7 +339,7 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
       }
       if (ok) {
 #pragma unroll
-        for (int h = 0; h < HALVES; ++h) Epi::end_unit(ep, st[h], row0 + h * kBM, split);
+        for (int h = 0; h < HALVES; ++h) Epi::end_unit(ep, st[h], row0 + h * kBM, split * G + grp);
       }
     }
     if (!ok) {

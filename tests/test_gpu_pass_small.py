@@ -78,7 +78,9 @@ def test_forward_with_fewer_vocabulary_partials(name):
     full = B.ps_lmhead_ppo_fwd_workspace_size(N, cfg.d, cfg.V, up.dcode)
     tiles = (cfg.V + 255) // 256
     for parts in (1, 3, tiles - 1):
-        small = full - 8 * N * (tiles - parts)   # exactly `parts` partials per row fit
+        # two 8-byte (max, sum) partials per row and vocabulary range (one per column group of the
+        # epilogue): exactly `parts` ranges fit
+        small = full - 16 * N * (tiles - parts)
         ws = torch.zeros(small, dtype=torch.uint8, device="cuda")
         outs = {k: torch.empty(N, device="cuda") for k in ("lse", "logp", "ratio", "coef", "row_loss")}
         loss = torch.zeros(1, dtype=torch.float64, device="cuda")

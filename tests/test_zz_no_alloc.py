@@ -52,7 +52,7 @@ def test_noalloc_forward_matches_workspace_forward_twice(name):
 
 
 def test_noalloc_rejects_problems_larger_than_its_scratch():
-    # 6 million rows need more than 64 MiB even with one partial per row: refused before any launch
+    # 6 million rows need more than 64 MiB even with one vocabulary range per row: refused before any launch
     # (the pointers are valid but never read).
     from paper_2606_29758_gb300 import _binding as B
     t = torch.zeros(64, device="cuda")
